@@ -1,0 +1,182 @@
+/*
+ * mc.h — C ABI of libmc: the fused LM-head log-prob / entropy forward, the
+ * MirrorPop sequence filter, and the fused backward, for one NVIDIA GB300
+ * (sm_103a).
+ *
+ * Every entry point takes plain pointers and sizes. Unless a parameter says
+ * "host", every pointer is DEVICE memory on the current CUDA device, owned by
+ * the caller, and must stay valid until the work queued on `stream` has
+ * finished. The library allocates no device memory: scratch comes in through
+ * `workspace` arguments sized by the matching *_workspace_size() query.
+ *
+ * Calls are stream-ordered and asynchronous. Errors that can be found on the
+ * host (null or misaligned pointers, bad sizes, a workspace that is too small,
+ * no sm_103 device) return a non-zero mc_status synchronously and queue no
+ * work. Errors found on the device (a target outside [0, V), a bounded wait
+ * that gave up) set bits of the caller's `dev_status` word (MC_DEV_* flags,
+ * never cleared by the library) and mark the affected outputs NaN.
+ *
+ * Layouts: matrices are row-major. hidden is [N, d] bf16, w_vocab is [V, d]
+ * bf16 (the LM head, one row per vocabulary entry), so the logits are
+ * z[t, v] = (hidden[t, :] . w_vocab[v, :]) * inv_temperature and are never
+ * written to memory. Row t's hidden state is the one that predicts targets[t]
+ * (the caller applies the usual one-token shift). Token arrays are packed
+ * over all sequences; cu_seqlens[B+1] gives the sequence boundaries.
+ *
+ * The paper: MusaCoder (arXiv 2606.04847). §4.4.1 Eq. 4 defines the token
+ * importance ratio, Eq. 5 the GRPO objective; §4.5.2 Eq. 17 the masked
+ * objective and Eq. 18-21 the sequence statistics and MirrorPop mask.
+ */
+#ifndef MC_H_
+#define MC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t (NULL = the legacy default stream). */
+typedef struct CUstream_st* mc_stream_t;
+
+typedef enum {
+  MC_OK = 0,
+  MC_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, size out of range */
+  MC_ERR_UNSUPPORTED = 2,   /* valid request this build does not run (e.g. d % 64 != 0, no sm_103 GPU) */
+  MC_ERR_CUDA = 3,          /* a CUDA runtime or driver call failed; see mc_last_cuda_error() */
+  MC_ERR_TIMEOUT = 4,       /* reported through dev_status: see MC_DEV_TIMEOUT */
+  MC_ERR_WORKSPACE = 5,     /* workspace pointer null/misaligned or smaller than the query */
+  MC_ERR_TARGET_RANGE = 6   /* reported through dev_status: see MC_DEV_TARGET_RANGE */
+} mc_status;
+
+/* Bits the kernels OR into *dev_status (an int32 in device memory). */
+#define MC_DEV_TIMEOUT      0x1  /* a bounded device-side wait gave up; outputs of that call are invalid */
+#define MC_DEV_TARGET_RANGE 0x2  /* some targets[t] was outside [0, V); those rows are NaN */
+
+/* Static text for a status code. */
+const char* mc_status_string(mc_status s);
+/* Text of the last CUDA error seen by this thread inside the library ("" if none). */
+const char* mc_last_cuda_error(void);
+/* ABI version: (major << 16) | minor. */
+int32_t mc_version(void);
+
+/* ------------------------------------------------------------------------
+ * Forward: per-token target log-prob, entropy and log-sum-exp.
+ *
+ * Computes, for every row t < N (pi_theta of Eq. 4 / Eq. 5, §4.4.1, taken as
+ * the softmax of the LM-head logits; the entropy is the Shannon entropy in
+ * nats of the same softmax, the diagnostic tracked in §5.4.6):
+ *   lse[t]     = log sum_v exp(z[t, v])
+ *   logp[t]    = z[t, targets[t]] - lse[t]
+ *   entropy[t] = -sum_v p log p,  p = exp(z[t, :] - lse[t])
+ * in one pass over the vocabulary (online max / sum / entropy update), fp32
+ * accumulation of bf16 products on the tensor cores.
+ *
+ *   hidden        bf16 [N, d], 16-byte aligned rows
+ *   w_vocab       bf16 [V, d], 16-byte aligned rows
+ *   targets       int32 [N]; a value outside [0, V) sets MC_DEV_TARGET_RANGE and
+ *                 makes that row's logp, entropy and lse NaN
+ *   N             rows, 0 <= N < 2^31 (N == 0 queues nothing and returns MC_OK)
+ *   d             hidden size, a positive multiple of 64, <= 16384
+ *   V             vocabulary size, 1 <= V < 2^31
+ *   inv_temperature  1/tau > 0 (tau = sampling temperature; 1 for none)
+ *   logp          fp32 [N] out
+ *   entropy, lse  fp32 [N] out, each may be NULL
+ *   workspace     device scratch of >= mc_token_logprobs_workspace_size(N, d, V)
+ *                 bytes, 256-byte aligned; contents on entry are ignored
+ *   dev_status    int32 [1] (may be NULL): MC_DEV_* bits are ORed in
+ * ------------------------------------------------------------------------ */
+size_t mc_token_logprobs_workspace_size(int64_t N, int32_t d, int32_t V);
+
+mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32_t* targets,
+                            int64_t N, int32_t d, int32_t V, float inv_temperature,
+                            float* logp, float* entropy, float* lse,
+                            void* workspace, size_t workspace_bytes,
+                            int32_t* dev_status, mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Backward of the forward above.
+ *
+ * For upstream gradients g[t] = dL/dlogp[t] and gH[t] = dL/dentropy[t]
+ * (gH may be NULL = 0), with p = exp(z - lse):
+ *   dZ[t, v]        = inv_temperature * ( g[t] (1[v = targets[t]] - p[t, v])
+ *                                         - gH[t] p[t, v] (log p[t, v] + entropy[t]) )
+ *   grad_hidden     = dZ . w_vocab           bf16 [N, d] (overwritten)
+ *   grad_w          = dZ^T . hidden          fp32 [V, d] (overwritten, or added to
+ *                                            when accumulate != 0)
+ * This is the gradient of the log-prob and entropy with respect to the LM-head
+ * inputs, which the masked GRPO objective (Eq. 17, §4.5.2) reaches through
+ * rho (Eq. 4). Rows with g[t] == 0 and gH[t] == 0 (tokens of sequences that
+ * MirrorPop dropped, masked tokens) contribute nothing and are skipped: their
+ * grad_hidden rows are written as zero. The logits are recomputed per tile
+ * on the tensor cores and never stored; dZ (a gradient) is staged in bf16 in
+ * the workspace.
+ *
+ *   lse, entropy  fp32 [N] from the forward (entropy may be NULL when gH is NULL)
+ *   grad_logp     fp32 [N]; grad_entropy fp32 [N] or NULL
+ *   workspace     >= mc_token_logprobs_bwd_workspace_size(N, d, V, 128) bytes;
+ *                 more workspace lets the rows run in fewer, larger chunks
+ *                 (mc_token_logprobs_bwd_workspace_size(N, d, V, N) = one chunk)
+ *   Other arguments as for the forward. A target outside [0, V) sets
+ *   MC_DEV_TARGET_RANGE; that row's gradient terms are dropped.
+ * ------------------------------------------------------------------------ */
+size_t mc_token_logprobs_bwd_workspace_size(int64_t N, int32_t d, int32_t V, int64_t rows_per_chunk);
+
+mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const int32_t* targets,
+                                const float* lse, const float* entropy,
+                                const float* grad_logp, const float* grad_entropy,
+                                int64_t N, int32_t d, int32_t V, float inv_temperature,
+                                void* grad_hidden, float* grad_w, int32_t accumulate,
+                                void* workspace, size_t workspace_bytes,
+                                int32_t* dev_status, mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Sequence importance-ratio statistics and the MirrorPop keep-mask.
+ *
+ * With log rho[t] = logp_policy[t] - logp_behaviour[t] (Eq. 4: policy over
+ * rollout/behaviour) and T_i = { t in [cu_seqlens[i], cu_seqlens[i+1]) :
+ * loss_mask[t] != 0 }, L_i = |T_i|:
+ *   n_tokens[i]    = L_i
+ *   signed_mean[i] = (1/L_i) sum_{T_i} log rho      (exponent of Eq. 18)
+ *   abs_mean[i]    = (1/L_i) sum_{T_i} |log rho|    (exponent of Eq. 20)
+ *   keep[i]        = abs_mean[i] <= delta           (Eq. 21)
+ *   keep_vanilla[i]= |signed_mean[i]| <= delta_vanilla (the conventional
+ *                    sequence mask, read as a symmetric log-space interval;
+ *                    0 when delta_vanilla < 0)
+ *   token_ratio[t] = exp(log rho[t])                (Eq. 4)
+ *   token_keep[t]  = keep[seq(t)] && loss_mask[t]
+ * A sequence with L_i = 0 gets signed_mean = abs_mean = 0 and keep = 0.
+ *
+ *   logp_policy, logp_behaviour  fp32 [N]
+ *   loss_mask     uint8 [N] or NULL (= all tokens count)
+ *   cu_seqlens    int64 [B+1], cu[0] = 0, non-decreasing, cu[B] = N
+ *                 (checked on the device only as far as needed to stay in bounds:
+ *                 a segment is clamped to [0, N))
+ *   B             sequences, 1 <= B < 2^31;  N tokens, 0 <= N < 2^40
+ *   delta         MirrorPop threshold in log-ratio space, >= 0
+ *   signed_mean, abs_mean  fp32 [B] out; n_tokens int32 [B] out; keep uint8 [B] out
+ *   keep_vanilla  uint8 [B] out or NULL;  token_ratio fp32 [N] out or NULL;
+ *   token_keep    uint8 [N] out or NULL
+ * ------------------------------------------------------------------------ */
+mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behaviour,
+                              const uint8_t* loss_mask, const int64_t* cu_seqlens,
+                              int32_t B, int64_t N, float delta, float delta_vanilla,
+                              float* signed_mean, float* abs_mean, int32_t* n_tokens,
+                              uint8_t* keep, uint8_t* keep_vanilla,
+                              float* token_ratio, uint8_t* token_keep, mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Self-test of the bounded device wait used by every pipelined kernel: one
+ * CTA waits on a shared-memory barrier that nothing ever signals, gives up
+ * after `timeout_ns` nanoseconds (1e6 <= timeout_ns <= 1e10), sets
+ * MC_DEV_TIMEOUT in *dev_status and returns. Exercises the failure path
+ * without faulting or hanging the GPU. (No counterpart in the paper.)
+ * ------------------------------------------------------------------------ */
+mc_status mc_selftest_bounded_wait(int32_t* dev_status, int64_t timeout_ns, mc_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MC_H_ */

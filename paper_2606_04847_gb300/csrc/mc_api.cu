@@ -1,0 +1,398 @@
+// mc_api.cu — the C ABI declared in include/mc.h.
+//
+// Host side only: checks arguments (before touching CUDA, so a bad call never
+// launches anything), checks the device is an sm_103 part, lays out the
+// caller's workspace, encodes the TMA descriptors and queues the kernels on
+// the caller's stream. No device memory is allocated here.
+#include <atomic>
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "mc.h"
+#include "mc_internal.h"
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBN = 256;
+constexpr int kMaxSplits = 16;
+constexpr size_t kStatusBytes = 256;
+constexpr int kMaxDevices = 64;
+
+thread_local std::string g_last_cuda_error;
+
+mc_status cuda_fail(cudaError_t e, const char* what) {
+  g_last_cuda_error = std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+  return MC_ERR_CUDA;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ---- cached device attributes (the only state the library keeps)
+std::atomic<int> g_dev_sms[kMaxDevices];
+std::atomic<int> g_dev_cc[kMaxDevices];
+
+mc_status device_info(int* sms) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return MC_ERR_UNSUPPORTED;
+  int cc = g_dev_cc[dev].load(std::memory_order_relaxed);
+  int n = g_dev_sms[dev].load(std::memory_order_relaxed);
+  if (cc == 0) {
+    int major = 0, minor = 0;
+    if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    if ((e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    cc = major * 10 + minor;
+    g_dev_sms[dev].store(n, std::memory_order_relaxed);
+    g_dev_cc[dev].store(cc, std::memory_order_relaxed);
+  }
+  if (cc != 103) return MC_ERR_UNSUPPORTED;  // kernels are built for sm_103a only
+  *sms = n;
+  return MC_OK;
+}
+
+uint64_t wait_timeout_ns() {
+  static const uint64_t t = [] {
+    const char* s = std::getenv("MC_WAIT_TIMEOUT_NS");
+    if (s != nullptr) {
+      const unsigned long long v = std::strtoull(s, nullptr, 10);
+      if (v >= 1000000ull && v <= 60000000000ull) return static_cast<uint64_t>(v);
+    }
+    return static_cast<uint64_t>(4000000000ull);  // 4 s: far above any healthy wait
+  }();
+  return t;
+}
+
+// ---- TMA descriptors
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<EncodeFn>(nullptr);
+    return reinterpret_cast<EncodeFn>(p);
+  }();
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] with row stride `stride_elems`, 128-byte
+// swizzled boxes of {64, box_outer}; out-of-range elements read as zero.
+mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_elems,
+                    uint32_t box_outer) {
+  EncodeFn fn = encode_fn();
+  if (fn == nullptr) {
+    g_last_cuda_error = "cuTensorMapEncodeTiled not available from the driver";
+    return MC_ERR_CUDA;
+  }
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {stride_elems * 2};
+  const cuuint32_t box[2] = {64, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char buf[128];
+    std::snprintf(buf, sizeof buf, "cuTensorMapEncodeTiled failed (CUresult %d)", static_cast<int>(r));
+    g_last_cuda_error = buf;
+    return MC_ERR_CUDA;
+  }
+  return MC_OK;
+}
+
+// Vocabulary tile ranges per 128-row block. Enough units to spread over the
+// SMs for small N, and at least 8 so the CTAs running together share few row
+// blocks (their hidden rows stay in L2) for large N.
+int choose_splits(long long m_blocks, int n_tiles, int sms) {
+  long long s = ceil_div(2LL * sms, m_blocks);
+  if (s < 8) s = 8;
+  if (s > kMaxSplits) s = kMaxSplits;
+  if (s > n_tiles) s = n_tiles;
+  return static_cast<int>(s < 1 ? 1 : s);
+}
+
+int max_splits(int V) {
+  const int n_tiles = static_cast<int>(ceil_div(V, kBN));
+  return n_tiles < kMaxSplits ? n_tiles : kMaxSplits;
+}
+
+bool valid_common(int64_t N, int32_t d, int32_t V, float inv_temperature) {
+  if (N < 0 || N >= (1LL << 31)) return false;
+  if (V < 1) return false;
+  if (d <= 0 || d % 64 != 0 || d > 16384) return false;
+  if (!(inv_temperature > 0.f) || !std::isfinite(inv_temperature)) return false;
+  return true;
+}
+
+struct FwdLayout {
+  size_t status_off, part_off, zy_off, total;
+  long long n_pad;
+};
+
+FwdLayout fwd_layout(int64_t N, int32_t V) {
+  FwdLayout L;
+  L.n_pad = ceil_div(N, kBM) * kBM;
+  const size_t part_bytes = size_t(3) * max_splits(V) * size_t(L.n_pad) * 4;
+  L.status_off = 0;
+  L.part_off = kStatusBytes;
+  L.zy_off = align_up(L.part_off + part_bytes, 256);
+  L.total = align_up(L.zy_off + size_t(L.n_pad) * 4, 256);
+  return L;
+}
+
+long long v_pad(int32_t V) { return ceil_div(V, 64) * 64; }
+
+}  // namespace
+
+extern "C" {
+
+const char* mc_status_string(mc_status s) {
+  switch (s) {
+    case MC_OK: return "MC_OK";
+    case MC_ERR_INVALID_ARG: return "MC_ERR_INVALID_ARG: invalid argument (null/misaligned pointer or size out of range)";
+    case MC_ERR_UNSUPPORTED: return "MC_ERR_UNSUPPORTED: unsupported shape or device (needs sm_103, d % 64 == 0)";
+    case MC_ERR_CUDA: return "MC_ERR_CUDA: a CUDA call failed (see mc_last_cuda_error)";
+    case MC_ERR_TIMEOUT: return "MC_ERR_TIMEOUT: a bounded device wait gave up";
+    case MC_ERR_WORKSPACE: return "MC_ERR_WORKSPACE: workspace missing, misaligned or too small";
+    case MC_ERR_TARGET_RANGE: return "MC_ERR_TARGET_RANGE: a target index outside [0, V)";
+  }
+  return "unknown mc_status";
+}
+
+const char* mc_last_cuda_error(void) { return g_last_cuda_error.c_str(); }
+
+int32_t mc_version(void) { return (1 << 16) | 0; }
+
+size_t mc_token_logprobs_workspace_size(int64_t N, int32_t d, int32_t V) {
+  if (!valid_common(N, d, V, 1.f)) return 0;
+  return fwd_layout(N, V).total;
+}
+
+mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32_t* targets, int64_t N,
+                            int32_t d, int32_t V, float inv_temperature, float* logp, float* entropy,
+                            float* lse, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                            mc_stream_t stream) {
+  if (!valid_common(N, d, V, inv_temperature)) return MC_ERR_INVALID_ARG;
+  if (N == 0) return MC_OK;
+  if (!hidden || !w_vocab || !targets || !logp) return MC_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(w_vocab, 16) || !aligned(targets, 4) || !aligned(logp, 4) ||
+      (entropy && !aligned(entropy, 4)) || (lse && !aligned(lse, 4)) || (dev_status && !aligned(dev_status, 4)))
+    return MC_ERR_INVALID_ARG;
+  const FwdLayout L = fwd_layout(N, V);
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < L.total) return MC_ERR_WORKSPACE;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  mc::FwdArgs a;
+  if ((st = make_tmap(&a.tm_hidden, hidden, d, N, d, kBM)) != MC_OK) return st;
+  if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, kBN)) != MC_OK) return st;
+  const long long m_blocks = ceil_div(N, kBM);
+  const int n_tiles = static_cast<int>(ceil_div(V, kBN));
+  a.targets = targets;
+  a.N = N;
+  a.d = d;
+  a.V = V;
+  a.inv_temperature = inv_temperature;
+  a.splits = choose_splits(m_blocks, n_tiles, sms);
+  a.n_pad = L.n_pad;
+  a.part = reinterpret_cast<float*>(ws + L.part_off);
+  a.zy = reinterpret_cast<float*>(ws + L.zy_off);
+  a.ws_status = reinterpret_cast<int32_t*>(ws + L.status_off);
+  a.logp = logp;
+  a.entropy = entropy;
+  a.lse = lse;
+  a.dev_status = dev_status;
+  a.grid = sms;
+  a.timeout_ns = wait_timeout_ns();
+  cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  e = mc::launch_forward(a, s);
+  if (e != cudaSuccess) return cuda_fail(e, "forward launch");
+  return MC_OK;
+}
+
+size_t mc_token_logprobs_bwd_workspace_size(int64_t N, int32_t d, int32_t V, int64_t rows_per_chunk) {
+  if (!valid_common(N, d, V, 1.f) || rows_per_chunk < 1) return 0;
+  long long r = rows_per_chunk < N ? rows_per_chunk : N;
+  r = ceil_div(r < 1 ? 1 : r, kBM) * kBM;
+  return kStatusBytes + align_up(size_t(r) * size_t(v_pad(V)) * 2, 256);
+}
+
+mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const int32_t* targets, const float* lse,
+                                const float* entropy, const float* grad_logp, const float* grad_entropy, int64_t N,
+                                int32_t d, int32_t V, float inv_temperature, void* grad_hidden, float* grad_w,
+                                int32_t accumulate, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                                mc_stream_t stream) {
+  if (!valid_common(N, d, V, inv_temperature)) return MC_ERR_INVALID_ARG;
+  if (!grad_w || !aligned(grad_w, 16)) return MC_ERR_INVALID_ARG;
+  if (N > 0) {
+    if (!hidden || !w_vocab || !targets || !lse || !grad_logp || !grad_hidden) return MC_ERR_INVALID_ARG;
+    if (grad_entropy && !entropy) return MC_ERR_INVALID_ARG;
+    if (!aligned(hidden, 16) || !aligned(w_vocab, 16) || !aligned(grad_hidden, 16) || !aligned(targets, 4) ||
+        !aligned(lse, 4) || !aligned(grad_logp, 4) || (entropy && !aligned(entropy, 4)) ||
+        (grad_entropy && !aligned(grad_entropy, 4)) || (dev_status && !aligned(dev_status, 4)))
+      return MC_ERR_INVALID_ARG;
+  }
+  const long long vp = v_pad(V);
+  long long R = 0;
+  if (N > 0) {
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < mc_token_logprobs_bwd_workspace_size(N, d, V, kBM))
+      return MC_ERR_WORKSPACE;
+    R = static_cast<long long>((workspace_bytes - kStatusBytes) / (size_t(vp) * 2));
+    R = R / kBM * kBM;
+    const long long n_pad = ceil_div(N, kBM) * kBM;
+    if (R > n_pad) R = n_pad;
+    if (R < kBM) return MC_ERR_WORKSPACE;
+  }
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (N == 0) {
+    if (!accumulate) {
+      e = cudaMemsetAsync(grad_w, 0, size_t(V) * size_t(d) * sizeof(float), s);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    }
+    return MC_OK;
+  }
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int32_t* ws_status = reinterpret_cast<int32_t*>(ws);
+  void* dz = ws + kStatusBytes;
+  e = cudaMemsetAsync(ws_status, 0, sizeof(int32_t), s);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+
+  CUtensorMap tm_w_k, tm_w_mn;
+  if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, kBN)) != MC_OK) return st;
+  if ((st = make_tmap(&tm_w_mn, w_vocab, d, V, d, 64)) != MC_OK) return st;
+  const int n_tiles = static_cast<int>(ceil_div(V, kBN));
+  const uint64_t tmo = wait_timeout_ns();
+  const uint16_t* h16 = static_cast<const uint16_t*>(hidden);
+  uint16_t* gh16 = static_cast<uint16_t*>(grad_hidden);
+
+  for (long long r0 = 0; r0 < N; r0 += R) {
+    const long long rows = (N - r0) < R ? (N - r0) : R;
+    const void* h_chunk = h16 + r0 * d;
+    mc::DzArgs za;
+    if ((st = make_tmap(&za.tm_hidden, h_chunk, d, rows, d, kBM)) != MC_OK) return st;
+    za.tm_w = tm_w_k;
+    za.targets = targets + r0;
+    za.lse = lse + r0;
+    za.entropy = entropy ? entropy + r0 : nullptr;
+    za.grad_logp = grad_logp + r0;
+    za.grad_entropy = grad_entropy ? grad_entropy + r0 : nullptr;
+    za.rows = rows;
+    za.d = d;
+    za.V = V;
+    za.inv_temperature = inv_temperature;
+    za.splits = choose_splits(ceil_div(rows, kBM), n_tiles, sms);
+    za.dz = dz;
+    za.ld = vp;
+    za.ws_status = ws_status;
+    za.grid = sms;
+    za.timeout_ns = tmo;
+    if ((e = mc::launch_dz(za, s)) != cudaSuccess) return cuda_fail(e, "dZ launch");
+
+    mc::DhArgs ha;
+    if ((st = make_tmap(&ha.tm_dz, dz, V, rows, vp, kBM)) != MC_OK) return st;
+    ha.tm_w_mn = tm_w_mn;
+    ha.rows = rows;
+    ha.d = d;
+    ha.V = V;
+    ha.grad_hidden = gh16 + r0 * d;
+    ha.ws_status = ws_status;
+    ha.grid = sms;
+    ha.timeout_ns = tmo;
+    if ((e = mc::launch_dh(ha, s)) != cudaSuccess) return cuda_fail(e, "dH launch");
+
+    mc::DwArgs wa;
+    if ((st = make_tmap(&wa.tm_dz_mn, dz, V, rows, vp, 64)) != MC_OK) return st;
+    if ((st = make_tmap(&wa.tm_h_mn, h_chunk, d, rows, d, 64)) != MC_OK) return st;
+    wa.rows = rows;
+    wa.d = d;
+    wa.V = V;
+    wa.grad_w = grad_w;
+    wa.accumulate = (accumulate || r0 > 0) ? 1 : 0;
+    wa.ws_status = ws_status;
+    wa.grid = sms;
+    wa.timeout_ns = tmo;
+    if ((e = mc::launch_dw(wa, s)) != cudaSuccess) return cuda_fail(e, "dW launch");
+  }
+  if ((e = mc::launch_status_merge(ws_status, dev_status, s)) != cudaSuccess) return cuda_fail(e, "status launch");
+  return MC_OK;
+}
+
+mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behaviour, const uint8_t* loss_mask,
+                              const int64_t* cu_seqlens, int32_t B, int64_t N, float delta, float delta_vanilla,
+                              float* signed_mean, float* abs_mean, int32_t* n_tokens, uint8_t* keep,
+                              uint8_t* keep_vanilla, float* token_ratio, uint8_t* token_keep, mc_stream_t stream) {
+  if (B < 1 || N < 0 || N >= (1LL << 40)) return MC_ERR_INVALID_ARG;
+  if (!(delta >= 0.f) || !std::isfinite(delta) || std::isnan(delta_vanilla)) return MC_ERR_INVALID_ARG;
+  if (!cu_seqlens || !signed_mean || !abs_mean || !n_tokens || !keep) return MC_ERR_INVALID_ARG;
+  if (N > 0 && (!logp_policy || !logp_behaviour)) return MC_ERR_INVALID_ARG;
+  if (!aligned(cu_seqlens, 8) || !aligned(signed_mean, 4) || !aligned(abs_mean, 4) || !aligned(n_tokens, 4) ||
+      (logp_policy && !aligned(logp_policy, 4)) || (logp_behaviour && !aligned(logp_behaviour, 4)) ||
+      (token_ratio && !aligned(token_ratio, 4)))
+    return MC_ERR_INVALID_ARG;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  mc::FilterArgs a;
+  a.logp_policy = logp_policy;
+  a.logp_behaviour = logp_behaviour;
+  a.loss_mask = loss_mask;
+  a.cu_seqlens = cu_seqlens;
+  a.B = B;
+  a.N = N;
+  a.delta = delta;
+  a.delta_vanilla = delta_vanilla;
+  a.signed_mean = signed_mean;
+  a.abs_mean = abs_mean;
+  a.n_tokens = n_tokens;
+  a.keep = keep;
+  a.keep_vanilla = keep_vanilla;
+  a.token_ratio = token_ratio;
+  a.token_keep = token_keep;
+  a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && (!token_ratio || aligned(token_ratio, 16)) &&
+             (!loss_mask || aligned(loss_mask, 4));
+  cudaError_t e = mc::launch_filter(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "filter launch");
+  return MC_OK;
+}
+
+mc_status mc_selftest_bounded_wait(int32_t* dev_status, int64_t timeout_ns, mc_stream_t stream) {
+  if (!dev_status || !aligned(dev_status, 4)) return MC_ERR_INVALID_ARG;
+  if (timeout_ns < 1000000LL || timeout_ns > 10000000000LL) return MC_ERR_INVALID_ARG;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  cudaError_t e = mc::launch_selftest_wait(dev_status, static_cast<uint64_t>(timeout_ns),
+                                           reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
+  return MC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,267 @@
+// mc_gemm.cuh — persistent warp-specialised tcgen05 GEMM engine for sm_103a.
+//
+// C[m, n] = sum_k A[m, k] B[n, k], bf16 operands, fp32 accumulation in TMEM.
+// The accumulator tile (BM x BN = 128 x 256) is handed to an epilogue functor
+// and never written to memory by the engine itself: the forward turns it into
+// an online log-sum-exp / entropy update, the backward into dZ, the backward
+// GEMMs into plain stores.
+//
+// CTA = 6 warps, one CTA per SM (the SMEM ring takes ~194 KB):
+//   warp 0        TMA producer: loads A/B k-blocks (BK = 64) into a 4-stage ring
+//   warp 1        TMEM allocator + MMA issuer (one thread): 4 x tcgen05.mma
+//                 (M=128, N=256, K=16) per k-block into one of two TMEM
+//                 accumulators (2 x 256 fp32 columns = all 512 columns)
+//   warps 2-5     epilogue: warp w reads TMEM lanes 32*(w%4)..+31, one output
+//                 row per thread, 32 columns per tcgen05.ld
+// The two accumulators let the epilogue of tile j overlap the MMAs of tile
+// j+1. Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a] per
+// accumulator. Every wait is bounded (mbar_wait), and on the way out each
+// role drains what it has in flight (TMA loads, MMAs) before TMEM is freed.
+//
+// Work decomposition: the M dimension is cut into BM-row blocks, the N
+// dimension into BN-column tiles, and the tiles of one row block into
+// `splits` contiguous ranges. A unit = (row block, range). Units are dealt
+// round-robin to the persistent CTAs (unit u -> CTA u % gridDim.x), so the
+// CTAs running at the same time share a few row blocks (A stays in L2) and
+// sweep the same B tiles together (B is read from HBM about once per wave).
+// Within a unit the tiles run in order, so an epilogue can carry per-row
+// state across them (the forward's online softmax).
+//
+// Operand layouts: A is [M, K] K-major (A_MN = false) or [K, M] M-major
+// (A_MN = true); B is [N, K] K-major or [K, N] N-major. All tiles use the
+// 128-byte swizzle; TMA boxes are 64 elements (128 B) wide in the contiguous
+// dimension. K-major A: one box {64 k, 128 m}; M-major A: two boxes
+// {64 m, 64 k}; K-major B: one box {64 k, 256 n}; N-major B: four boxes
+// {64 n, 64 k}. Out-of-range rows/columns are zero-filled by TMA.
+#pragma once
+
+#include "mc_ptx.cuh"
+
+namespace mc {
+
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;
+constexpr int UMMA_K = 16;
+constexpr int NUM_STAGES = 4;
+constexpr int NUM_ACC = 2;
+constexpr int TMEM_COLS = NUM_ACC * BN;  // 512
+constexpr int A_STAGE_BYTES = BM * BK * 2;  // 16 KB
+constexpr int B_STAGE_BYTES = BN * BK * 2;  // 32 KB
+constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+constexpr int GEMM_THREADS = 192;
+constexpr int EPI_WARP_BEGIN = 2;
+constexpr int NUM_EPI_WARPS = 4;
+constexpr int MN_BOX_BYTES = 64 * 64 * 2;  // one {64, 64} bf16 box = 8 KB
+
+struct GemmShared {
+  uint64_t full[NUM_STAGES];
+  uint64_t empty[NUM_STAGES];
+  uint64_t tfull[NUM_ACC];
+  uint64_t tempty[NUM_ACC];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+constexpr size_t GEMM_SMEM_BYTES = size_t(NUM_STAGES) * STAGE_BYTES + sizeof(GemmShared) + 1024;
+
+struct Schedule {
+  int m_blocks;  // ceil(M / BM)
+  int n_tiles;   // ceil(N / BN)
+  int splits;    // tile ranges per row block, 1 <= splits <= n_tiles
+  int k_blocks;  // ceil(K / BK)
+
+  __device__ __forceinline__ int units() const { return m_blocks * splits; }
+  __device__ __forceinline__ void unit(int u, int& mb, int& split, int& t0, int& t1) const {
+    mb = u / splits;
+    split = u - mb * splits;
+    t0 = static_cast<int>((static_cast<long long>(split) * n_tiles) / splits);
+    t1 = static_cast<int>((static_cast<long long>(split + 1) * n_tiles) / splits);
+  }
+};
+
+// Epilogue functor contract (one instance per epilogue thread):
+//   struct Epi {
+//     struct Params;
+//     __device__ void begin(const Params&, long long row, int mb, int split);
+//     __device__ void tile(const Params&, long long row, int n_tile, uint32_t taddr);
+//     __device__ void end(const Params&, long long row, int mb, int split, bool ok);
+//   };
+// `row` = global M index of the thread's row (may be >= M: padding rows),
+// `taddr` = TMEM address of the thread's warp's lane quadrant, column 0 of the
+// accumulator holding tile `n_tile`. `ok` is false when the pipeline gave up.
+
+template <class Epi, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const Schedule sch, const typename Epi::Params ep, const uint64_t timeout_ns,
+                    int32_t* dev_status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  GemmShared* sh = reinterpret_cast<GemmShared*>(smem + NUM_STAGES * STAGE_BYTES);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+#pragma unroll
+    for (int s = 0; s < NUM_STAGES; ++s) {
+      mbar_init(&sh->full[s], 1);
+      mbar_init(&sh->empty[s], 1);
+    }
+#pragma unroll
+    for (int a = 0; a < NUM_ACC; ++a) {
+      mbar_init(&sh->tfull[a], 1);
+      mbar_init(&sh->tempty[a], NUM_EPI_WARPS);
+    }
+    mbar_init(&sh->drain, 1);
+    sh->abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sh->tmem_base, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sh->tmem_base;
+  volatile int* abort = &sh->abort;
+  const int n_units = sch.units();
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+      uint32_t it = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        int mb, split, t0, t1;
+        sch.unit(u, mb, split, t0, t1);
+        for (int t = t0; t < t1 && ok; ++t) {
+          for (int kb = 0; kb < sch.k_blocks; ++kb) {
+            const int s = static_cast<int>(it % NUM_STAGES);
+            const uint32_t ph = (it / NUM_STAGES) & 1u;
+            if (!mbar_wait(&sh->empty[s], ph ^ 1u, abort, timeout_ns, dev_status)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&sh->full[s], STAGE_BYTES);
+            uint8_t* a = smem + s * STAGE_BYTES;
+            uint8_t* b = a + A_STAGE_BYTES;
+            if (!A_MN) {
+              tma_load_2d(a, &tmA, &sh->full[s], kb * BK, mb * BM);
+            } else {
+#pragma unroll
+              for (int j = 0; j < BM / 64; ++j)
+                tma_load_2d(a + j * MN_BOX_BYTES, &tmA, &sh->full[s], mb * BM + j * 64, kb * BK);
+            }
+            if (!B_MN) {
+              tma_load_2d(b, &tmB, &sh->full[s], kb * BK, t * BN);
+            } else {
+#pragma unroll
+              for (int j = 0; j < BN / 64; ++j)
+                tma_load_2d(b + j * MN_BOX_BYTES, &tmB, &sh->full[s], t * BN + j * 64, kb * BK);
+            }
+            ++it;
+          }
+        }
+      }
+      // Let every load this thread issued land before the CTA can exit.
+      const uint32_t last = it < NUM_STAGES ? it : NUM_STAGES;
+      for (uint32_t j = it - last; j < it; ++j)
+        mbar_wait(&sh->full[j % NUM_STAGES], (j / NUM_STAGES) & 1u, nullptr, timeout_ns, dev_status);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN, A_MN, B_MN);
+      uint32_t it = 0, tc = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        int mb, split, t0, t1;
+        sch.unit(u, mb, split, t0, t1);
+        for (int t = t0; t < t1 && ok; ++t) {
+          const uint32_t acc = tc & 1u;
+          const uint32_t aph = (tc >> 1) & 1u;
+          if (!mbar_wait(&sh->tempty[acc], aph ^ 1u, abort, timeout_ns, dev_status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem + acc * BN;
+          for (int kb = 0; kb < sch.k_blocks; ++kb) {
+            const int s = static_cast<int>(it % NUM_STAGES);
+            const uint32_t ph = (it / NUM_STAGES) & 1u;
+            if (!mbar_wait(&sh->full[s], ph, abort, timeout_ns, dev_status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a_addr = smem_u32(smem + s * STAGE_BYTES);
+            const uint32_t b_addr = a_addr + A_STAGE_BYTES;
+#pragma unroll
+            for (int k = 0; k < BK / UMMA_K; ++k) {
+              const uint64_t adesc = A_MN ? smem_desc_sw128(a_addr + k * (UMMA_K * 128), MN_BOX_BYTES, 1024)
+                                          : smem_desc_sw128(a_addr + k * (UMMA_K * 2), 16, 1024);
+              const uint64_t bdesc = B_MN ? smem_desc_sw128(b_addr + k * (UMMA_K * 128), MN_BOX_BYTES, 1024)
+                                          : smem_desc_sw128(b_addr + k * (UMMA_K * 2), 16, 1024);
+              umma_bf16(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+            }
+            umma_commit(&sh->empty[s]);  // frees the stage once these MMAs have read it
+            ++it;
+          }
+          if (!ok) break;
+          umma_commit(&sh->tfull[acc]);  // accumulator ready for the epilogue
+          ++tc;
+        }
+      }
+      // No MMA may still be writing TMEM when it is freed.
+      umma_commit(&sh->drain);
+      mbar_wait(&sh->drain, 0, nullptr, timeout_ns, dev_status);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+    const int row_in_block = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t tc = 0;
+    Epi epi;
+    bool ok = true;
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      int mb, split, t0, t1;
+      sch.unit(u, mb, split, t0, t1);
+      const long long row = static_cast<long long>(mb) * BM + row_in_block;
+      epi.begin(ep, row, mb, split);
+      for (int t = t0; t < t1; ++t) {
+        const uint32_t acc = tc & 1u;
+        const uint32_t aph = (tc >> 1) & 1u;
+        // Every lane polls; the warp proceeds only if all lanes saw the phase
+        // complete, so the warp-collective tcgen05.ld below stays converged.
+        const bool got = mbar_wait(&sh->tfull[acc], aph, abort, timeout_ns, dev_status);
+        if (!__all_sync(0xffffffffu, got)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        epi.tile(ep, row, t, tmem + acc * BN + lane_off);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh->tempty[acc]);
+        ++tc;
+      }
+      epi.end(ep, row, mb, split, ok);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+}  // namespace mc

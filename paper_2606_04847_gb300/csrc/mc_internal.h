@@ -1,0 +1,107 @@
+// mc_internal.h — launch entry points shared between the kernel translation
+// units and the C-ABI layer (mc_api.cu). Not part of the public ABI.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace mc {
+
+// Forward: persistent tcgen05 kernel (online log-softmax epilogue) followed by
+// the per-row merge of the split partials.
+struct FwdArgs {
+  CUtensorMap tm_hidden;  // K-major {d, N}, box {64, 128}
+  CUtensorMap tm_w;       // K-major {d, V}, box {64, 256}
+  const int32_t* targets;
+  long long N;
+  int d, V;
+  float inv_temperature;
+  int splits;
+  long long n_pad;
+  float* part;            // workspace: [3][splits][n_pad]
+  float* zy;              // workspace: [n_pad]
+  int32_t* ws_status;     // workspace: internal status word (zeroed by the caller)
+  float* logp;
+  float* entropy;
+  float* lse;
+  int32_t* dev_status;
+  int grid;
+  uint64_t timeout_ns;
+};
+cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream);
+
+// Backward building blocks.
+struct DzArgs {
+  CUtensorMap tm_hidden;  // K-major {d, rows}, box {64, 128}
+  CUtensorMap tm_w;       // K-major {d, V}, box {64, 256}
+  const int32_t* targets;
+  const float* lse;
+  const float* entropy;
+  const float* grad_logp;
+  const float* grad_entropy;
+  long long rows;
+  int d, V;
+  float inv_temperature;
+  int splits;
+  void* dz;               // bf16 [rows, ld]
+  long long ld;
+  int32_t* ws_status;
+  int grid;
+  uint64_t timeout_ns;
+};
+cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream);
+
+struct DhArgs {           // grad_hidden[rows, d] = dZ[rows, V] . W[V, d]
+  CUtensorMap tm_dz;      // K-major {V, rows}, box {64, 128}
+  CUtensorMap tm_w_mn;    // N-major {d, V}, box {64, 64}
+  long long rows;
+  int d, V;
+  void* grad_hidden;      // bf16, row stride d
+  int32_t* ws_status;
+  int grid;
+  uint64_t timeout_ns;
+};
+cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream);
+
+struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . H[rows, d]
+  CUtensorMap tm_dz_mn;   // M-major {V, rows}, box {64, 64}
+  CUtensorMap tm_h_mn;    // N-major {d, rows}, box {64, 64}
+  long long rows;
+  int d, V;
+  float* grad_w;
+  int accumulate;
+  int32_t* ws_status;
+  int grid;
+  uint64_t timeout_ns;
+};
+cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream);
+
+// Propagates the internal status word to the caller's (if any).
+cudaError_t launch_status_merge(const int32_t* ws_status, int32_t* dev_status, cudaStream_t stream);
+
+struct FilterArgs {
+  const float* logp_policy;
+  const float* logp_behaviour;
+  const uint8_t* loss_mask;
+  const int64_t* cu_seqlens;
+  int B;
+  long long N;
+  float delta, delta_vanilla;
+  float* signed_mean;
+  float* abs_mean;
+  int32_t* n_tokens;
+  uint8_t* keep;
+  uint8_t* keep_vanilla;
+  float* token_ratio;
+  uint8_t* token_keep;
+  int vec_ok;             // all float arrays 16-byte and loss_mask 4-byte aligned
+};
+cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream);
+
+cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream);
+
+size_t gemm_smem_bytes();
+
+}  // namespace mc

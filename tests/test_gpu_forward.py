@@ -1,0 +1,121 @@
+"""GPU forward (mc_token_logprobs) vs the fp64 oracle, element by element.
+
+Sizes span several 128-row blocks and 256-column vocabulary tiles, with
+ragged tails in both, the tiny config at full size, and the edge cases:
+N = 1, V not a multiple of the tile, V < one tile, targets at 0 and V-1,
+peaked softmax (low entropy), temperature, d = 64 and d = 5120.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import TOL_ENT, TOL_LOGP, assert_close_abs, np_
+from paper_2606_04847_gb300 import mc, workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def run_and_compare(wl, inv_temp=1.0, targets=None):
+    h = wl.hidden.cuda()
+    w = wl.w_vocab.cuda()
+    y = (wl.targets if targets is None else targets).cuda()
+    out = mc.token_logprobs(h, w, y, inv_temp)
+    torch.cuda.synchronize()
+    ref = oracle.token_logprobs(wl.hidden, wl.w_vocab, y.cpu(), inv_temp)
+    assert_close_abs(np_(out["logp"]), ref["logp"], TOL_LOGP, "logp")
+    assert_close_abs(np_(out["entropy"]), ref["entropy"], TOL_ENT, "entropy")
+    assert_close_abs(np_(out["lse"]), ref["lse"], TOL_LOGP, "lse")
+    return out, ref
+
+
+def test_config1_tiny_full_size():
+    wl = workloads.build(workloads.spec_for(1), "cpu")
+    run_and_compare(wl)
+
+
+@pytest.mark.parametrize("N,d,V", [
+    (1, 64, 300),            # single row, V < 2 tiles with a tail
+    (300, 128, 4097),        # ragged rows (3 blocks) and one-column vocab tail
+    (129, 256, 200),         # V smaller than one tile
+    (520, 512, 151936 // 16),  # 9496 = 37 tiles + 24 columns
+    (257, 5120, 1024),       # the 27B-class hidden size
+])
+def test_ragged_shapes(N, d, V):
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=d, V=V)
+    run_and_compare(workloads.build(spec, "cpu"))
+
+
+def test_targets_at_vocab_edges_and_temperature():
+    spec = workloads.spec_for(1, n_seqs=2, len_lo=150, len_hi=150, d=256, V=1000)
+    wl = workloads.build(spec, "cpu")
+    y = wl.targets.clone()
+    y[::3] = 0
+    y[1::3] = 999
+    run_and_compare(wl, inv_temp=1.0 / 0.9, targets=y)
+
+
+def test_peaked_softmax_low_entropy():
+    """W scaled x8: logits std ~8, entropies spread over ~[0, 3] nats."""
+    spec = workloads.spec_for(1, n_seqs=2, len_lo=200, len_hi=200, d=512, V=3000, w_scale=8.0)
+    out, ref = run_and_compare(workloads.build(spec, "cpu"))
+    assert ref["entropy"].min() < 0.5
+
+
+def test_uniform_logits():
+    """W = 0: every logit equal; logp = -log V and entropy = log V."""
+    N, d, V = 130, 64, 777
+    h = torch.randn(N, d).to(torch.bfloat16).cuda()
+    w = torch.zeros(V, d, dtype=torch.bfloat16).cuda()
+    y = torch.randint(0, V, (N,), dtype=torch.int32).cuda()
+    out = mc.token_logprobs(h, w, y)
+    assert_close_abs(np_(out["logp"]), np.full(N, -math.log(V)), 1e-5, "logp")
+    assert_close_abs(np_(out["entropy"]), np.full(N, math.log(V)), 1e-4, "entropy")
+
+
+def test_out_of_range_target_sets_status_and_nan():
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=40, len_hi=40, d=64, V=500)
+    wl = workloads.build(spec, "cpu")
+    y = wl.targets.clone()
+    y[3] = 500
+    y[7] = -1
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = mc.token_logprobs(wl.hidden.cuda(), wl.w_vocab.cuda(), y.cuda(), dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & mc.MC_DEV_TARGET_RANGE
+    lp = np_(out["logp"])
+    assert np.isnan(lp[3]) and np.isnan(lp[7])
+    good = np.ones(40, dtype=bool)
+    good[[3, 7]] = False
+    ref = oracle.token_logprobs(wl.hidden, wl.w_vocab, wl.targets)
+    assert_close_abs(lp[good], ref["logp"][good], TOL_LOGP, "logp of valid rows")
+
+
+def test_deterministic_bitwise():
+    wl = workloads.build(workloads.spec_for(1, n_seqs=3, len_lo=100, len_hi=100, d=512, V=5000), "cpu")
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    a = mc.token_logprobs(h, w, y)
+    b = mc.token_logprobs(h, w, y)
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_nullable_outputs_and_zero_rows():
+    wl = workloads.build(workloads.spec_for(1, n_seqs=1, len_lo=64, len_hi=64, d=64, V=256), "cpu")
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    full = mc.token_logprobs(h, w, y)
+    only = mc.token_logprobs(h, w, y, out={"logp": torch.empty(64, device="cuda")})
+    assert torch.equal(full["logp"], only["logp"])
+    empty = mc.token_logprobs(h[:0], w, y[:0])
+    assert empty["logp"].numel() == 0
+
+
+def test_bounded_wait_selftest_keeps_context_usable():
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    mc.selftest_bounded_wait(st, 20_000_000)  # 20 ms
+    torch.cuda.synchronize()
+    assert int(st.item()) & mc.MC_DEV_TIMEOUT
+    test_config1_tiny_full_size()  # the context is still healthy
