@@ -1,0 +1,466 @@
+"""Throughput of the fused log-prob forward + MirrorPop filter + backward.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One step = one pass of the whole hot path over one batch of the 9B-class
+fused forward+backward workload (32 sequences of U[512, 8192] tokens, d = 4096,
+V = 248320, bf16; seeded synthetic inputs, see paper_2606_04847_gb300/workloads.py):
+  1. mc_token_logprobs      policy log-probs, entropies, log-sum-exp
+  2. mc_seq_ratio_filter    per-sequence ratio statistics + MirrorPop keep-mask
+  3. mc_token_logprobs_bwd  grad_hidden, grad_w for advantage weights on the
+                            kept tokens (row_keep = the filter's token_keep)
+The behaviour log-probs are the policy's plus a per-sequence N(0, 0.2^2) gap,
+formed once before timing (the rollout engine's job, not part of the step).
+
+Rank 0 prints one JSON line. ``value`` = tokens/s over all ranks with inputs
+resident in HBM; ``e2e`` = the same through the C ABI with the step's inputs
+copied from pinned host memory and its per-token / per-sequence results read
+back inside the timed region. Inputs (hidden 1.1 GB, W 2.0 GB) exceed the
+129 MB L2, so no flush is needed between steps. ``--impl reference`` times the
+CPU fp64 oracle instead, on a bounded sample of the same workload.
+
+Multi-GPU (torchrun): one independent replica per GPU (each rank its own
+batch, weak scaling); the path shards with no data-path collective.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+METRIC = "rollout tokens/sec for fused logprob fwd+bwd at 1 GB300; % of bf16 tensor peak"
+CONFIG_ID = 5
+FWD_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fwd_kernel_traffic.json")
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"], "bf16_sustained": d["bf16_tflops_sustained"],
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+def _kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu"):
+        h.update(open(os.path.join(ROOT, "paper_2606_04847_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle reasons sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"mc_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None, "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def _dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def _barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def _max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _sum_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# --------------------------------------------------------------------------- CPU oracle leg
+
+
+def oracle_sample_step(wl, rows, delta):
+    """The fp64 oracle over the first `rows` packed tokens of the workload:
+    forward, filter (those tokens as one sequence), backward with the kept
+    advantage weights. Returns elapsed seconds."""
+    import numpy as np
+
+    import oracle
+
+    h = wl.hidden[:rows].cpu()
+    w = wl.w_vocab.cpu() if wl.w_vocab.is_cuda else wl.w_vocab
+    y = wl.targets[:rows].cpu()
+    adv = wl.advantages[:rows].cpu().double().numpy()
+    gap = wl.gap[:rows].cpu().double().numpy()
+    t0 = time.perf_counter()
+    fw = oracle.token_logprobs(h, w, y, 1.0)
+    flt = oracle.seq_ratio_filter(fw["logp"], fw["logp"] + gap, None, np.array([0, rows]), delta, delta)
+    g = adv * flt["token_keep"]
+    oracle.token_logprobs_bwd(h, w, y, g, None, 1.0)
+    return time.perf_counter() - t0
+
+
+def _cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# --------------------------------------------------------------------------- main
+
+
+def run_ours(args):
+    from paper_2606_04847_gb300 import build as mcbuild
+    from paper_2606_04847_gb300 import mc, workloads
+
+    world, rank, local = _dist_setup(args)
+    if not os.path.exists(mc.lib_path()):
+        mcbuild.build()
+    spec = workloads.spec_for(CONFIG_ID)
+    if world > 1:
+        spec = workloads.spec_for(CONFIG_ID, seed=spec.seed + 1000 * rank)  # each replica its own batch
+    wl = workloads.build(spec, "cuda")
+    dev = torch.device("cuda")
+    N, d, V, B = wl.N, spec.d, spec.V, wl.B
+    delta = spec.delta
+    h, w, y = wl.hidden, wl.w_vocab, wl.targets
+    cu, mask, adv = wl.cu_seqlens, wl.loss_mask, wl.advantages
+
+    # Behaviour log-probs: policy log-probs + the per-sequence gap (untimed).
+    pre = mc.token_logprobs(h, w, y)
+    logp_b = (pre["logp"] + wl.gap).contiguous()
+    del pre
+
+    fw_out = {k: torch.empty(N, dtype=torch.float32, device=dev) for k in ("logp", "entropy", "lse")}
+    fw_ws = torch.empty(mc.forward_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
+    bw_ws = torch.empty(mc.backward_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
+    gh = torch.empty((N, d), dtype=torch.bfloat16, device=dev)
+    gw = torch.empty((V, d), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    ev = {k: [] for k in ("fwd", "filter", "bwd")}
+
+    def step(record=False, inputs=None):
+        hh, yy, lb, mm, cc, aa = inputs if inputs is not None else (h, y, logp_b, mask, cu, adv)
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)] if record else None
+        if record:
+            e[0].record(stream)
+        mc.token_logprobs(hh, w, yy, out=fw_out, workspace=fw_ws, stream=stream)
+        if record:
+            e[1].record(stream)
+        flt = mc.seq_ratio_filter(fw_out["logp"], lb, mm, cc, delta, delta, stream=stream)
+        if record:
+            e[2].record(stream)
+        mc.token_logprobs_bwd(hh, w, yy, fw_out["lse"], fw_out["entropy"], aa, None, row_keep=flt["token_keep"],
+                              grad_hidden=gh, grad_w=gw, workspace=bw_ws, stream=stream)
+        if record:
+            e[3].record(stream)
+            ev["fwd"].append((e[0], e[1]))
+            ev["filter"].append((e[1], e[2]))
+            ev["bwd"].append((e[2], e[3]))
+        return flt
+
+    for _ in range(args.warmup):
+        flt = step()
+    torch.cuda.synchronize()
+    kept_rows = int(flt["token_keep"].sum().item())
+    n_keep_seq = int(flt["keep"].sum().item())
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    _barrier(world)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        step(record=True)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    _barrier(world)
+    clk = clocks.stop()
+    ms = t_start.elapsed_time(t_end)
+    ms_max = _max_over_ranks(ms, world)
+    tokens_total = _sum_over_ranks(float(N) * args.steps, world)
+    value = tokens_total / (ms_max / 1e3)
+
+    def avg(k):
+        return sum(a.elapsed_time(b) for a, b in ev[k]) / len(ev[k])
+
+    t_fwd, t_flt, t_bwd = avg("fwd"), avg("filter"), avg("bwd")
+    flop_fwd = 2.0 * N * d * V
+    flop_bwd = 4.0 * kept_rows * d * V  # algorithmic: rows with a nonzero upstream gradient
+    peaks = _peaks()
+    peak_tf = peaks["bf16_sustained"]
+    achieved = flop_fwd / (t_fwd / 1e3) / 1e12
+    traffic = None
+    if os.path.exists(FWD_TRAFFIC_FILE):
+        tj = json.load(open(FWD_TRAFFIC_FILE))
+        if tj.get("kernel_source_hash") == _kernel_source_hash():
+            traffic = tj["bytes_per_full_launch"] * (N / tj["full_launch_rows"])
+    step_tflops = (flop_fwd + flop_bwd) * args.steps / (ms / 1e3) / 1e12
+
+    # ---------------------------------------------------------------- e2e through the C ABI, host buffers
+    e2e = None
+    if not args.no_e2e:
+        host = [t.cpu().pin_memory() for t in (h, y, logp_b, mask, cu, adv)]
+        dev_in = [torch.empty_like(t, device=dev) for t in host]
+        outs_d = None
+        host_out = None
+        h2d = sum(t.numel() * t.element_size() for t in host)
+        for i in range(2):  # warm
+            for dst, src in zip(dev_in, host):
+                dst.copy_(src, non_blocking=True)
+            f = step(inputs=dev_in)
+        torch.cuda.synchronize()
+        outs_d = [fw_out["logp"], fw_out["entropy"], f["signed_mean"], f["abs_mean"], f["n_tokens"], f["keep"],
+                  f["token_keep"]]
+        host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs_d]
+        d2h = sum(t.numel() * t.element_size() for t in host_out)
+        _barrier(world)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            for dst, src in zip(dev_in, host):
+                dst.copy_(src, non_blocking=True)
+            f = step(inputs=dev_in)
+            outs_d = [fw_out["logp"], fw_out["entropy"], f["signed_mean"], f["abs_mean"], f["n_tokens"],
+                      f["keep"], f["token_keep"]]
+            for dst, src in zip(host_out, outs_d):
+                dst.copy_(src, non_blocking=True)
+        b.record(stream)
+        torch.cuda.synchronize()
+        _barrier(world)
+        e2e_ms = _max_over_ranks(a.elapsed_time(b), world)
+        e2e = {"value": tokens_total / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    # ---------------------------------------------------------------- CPU oracle baseline (rank 0, N = 1)
+    cpu = None
+    if world == 1 and not args.no_cpu:
+        rows = args.cpu_rows
+        secs = oracle_sample_step(wl, rows, delta)
+        cpu = {"value": rows / secs, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+               "sample": f"first {rows} packed tokens of the workload (one sequence slice): fp64 forward over "
+                         f"V={V}, filter, backward; {secs:.1f} s"}
+
+    launches_per_step = 2 + 1 + 5  # forward + finalize; filter; select, gather, dZ, dH, dW (one chunk)
+    if rank == 0:
+        line = {
+            "metric": METRIC,
+            "value": value,
+            "unit": "tokens/s",
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": ms_max / args.steps,
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": spec.name, "tokens_per_step": N, "sequences": B, "d": d, "V": V,
+                       "delta": delta, "kept_sequences": n_keep_seq, "kept_tokens": kept_rows,
+                       "l2": "inputs larger than L2 (hidden 1.1 GB, W 2.0 GB); no flush",
+                       "parallelism": f"replicas x{world}"},
+            "pct_of_bf16_peak": step_tflops / peak_tf,
+            "step_tflops_algorithmic": step_tflops,
+            "ms_by_call": {"forward": t_fwd, "filter": t_flt, "backward": t_bwd},
+            "clocks": clk,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps,
+            "roofline": {"bound": "tensor", "kernel": "forward (tcgen05 projection + online log-softmax)",
+                         "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s", "frac": achieved / peak_tf,
+                         "peak_source": f"{peaks['source']} bf16 sustained", "traffic": traffic},
+            "roofline_backward": {"bound": "tensor", "achieved": flop_bwd / (t_bwd / 1e3) / 1e12,
+                                  "peak": peak_tf, "unit": "TFLOP/s",
+                                  "frac": flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf},
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def run_case(args):
+    """One call of the path, `--launches` times, for ncu captures (no timing printed
+    beyond a one-line summary): --case fwd|bwd|filter on the first `--rows`
+    tokens of the workload (0 = all)."""
+    from paper_2606_04847_gb300 import build as mcbuild
+    from paper_2606_04847_gb300 import mc, workloads
+
+    torch.cuda.set_device(0)
+    if not os.path.exists(mc.lib_path()):
+        mcbuild.build()
+    spec = workloads.spec_for(CONFIG_ID)
+    wl = workloads.build(spec, "cuda")
+    R = wl.N if args.rows <= 0 else min(args.rows, wl.N)
+    h, w, y = wl.hidden[:R].contiguous(), wl.w_vocab, wl.targets[:R].contiguous()
+    fw = mc.token_logprobs(h, w, y)
+    cu = torch.tensor([0, R], dtype=torch.int64, device="cuda")
+    lb = (fw["logp"] + wl.gap[:R]).contiguous()
+    flt = mc.seq_ratio_filter(fw["logp"], lb, None, cu, spec.delta, spec.delta)
+    adv = wl.advantages[:R].contiguous()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.launches):
+        if args.case == "fwd":
+            mc.token_logprobs(h, w, y, out=fw)
+        elif args.case == "filter":
+            mc.seq_ratio_filter(fw["logp"], lb, None, cu, spec.delta, spec.delta)
+        else:
+            mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], adv, None, row_keep=flt["token_keep"])
+    torch.cuda.synchronize()
+    print(json.dumps({"case": args.case, "rows": R, "launches": args.launches,
+                      "wall_ms_per_launch": (time.perf_counter() - t0) * 1e3 / args.launches}))
+
+
+def run_reference(args):
+    """The CPU fp64 oracle, as it stands, on a bounded sample per step."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2606_04847_gb300 import workloads
+
+    spec = workloads.spec_for(CONFIG_ID)
+    wl = workloads.build(spec, "cuda" if torch.cuda.is_available() else "cpu")
+    rows = args.ref_rows
+    for _ in range(args.warmup):
+        oracle_sample_step(wl, rows, spec.delta)
+    total = 0.0
+    for _ in range(args.steps):
+        total += oracle_sample_step(wl, rows, spec.delta)
+    value = rows * args.steps / total
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": value,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": total / args.steps * 1e3,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": spec.name, "tokens_per_step": rows, "d": spec.d, "V": spec.V,
+                   "note": "each step: the oracle on the first packed tokens of the workload"},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+                         "sample": f"{rows} tokens per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-rows", type=int, default=32)
+    ap.add_argument("--ref-rows", type=int, default=8)
+    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter"], default="step",
+                    help="profiling aid: run one call of the path --launches times")
+    ap.add_argument("--rows", type=int, default=0, help="--case: tokens to use (0 = the whole batch)")
+    ap.add_argument("--launches", type=int, default=2)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    elif args.case != "step":
+        run_case(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -107,9 +107,11 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
  *                                            when accumulate != 0)
  * This is the gradient of the log-prob and entropy with respect to the LM-head
  * inputs, which the masked GRPO objective (Eq. 17, §4.5.2) reaches through
- * rho (Eq. 4). Rows with g[t] == 0 and gH[t] == 0 (tokens of sequences that
- * MirrorPop dropped, masked tokens) contribute nothing and are skipped: their
- * grad_hidden rows are written as zero. The logits are recomputed per tile
+ * rho (Eq. 4). Eq. 17 multiplies every token of response i by its mask M_i:
+ * `row_keep` (uint8 [N], nullable = all kept) applies that gate, so
+ * g[t] and gH[t] count only where row_keep[t] != 0 (pass the filter's
+ * token_keep). Rows with a zero effective upstream gradient contribute
+ * nothing: their grad_hidden rows are written as zero. The logits are recomputed per tile
  * on the tensor cores and never stored; dZ (a gradient) is staged in bf16 in
  * the workspace.
  *
@@ -126,7 +128,7 @@ size_t mc_token_logprobs_bwd_workspace_size(int64_t N, int32_t d, int32_t V, int
 mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const int32_t* targets,
                                 const float* lse, const float* entropy,
                                 const float* grad_logp, const float* grad_entropy,
-                                int64_t N, int32_t d, int32_t V, float inv_temperature,
+                                const uint8_t* row_keep, int64_t N, int32_t d, int32_t V, float inv_temperature,
                                 void* grad_hidden, float* grad_w, int32_t accumulate,
                                 void* workspace, size_t workspace_bytes,
                                 int32_t* dev_status, mc_stream_t stream);

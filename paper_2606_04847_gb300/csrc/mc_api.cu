@@ -162,6 +162,24 @@ FwdLayout fwd_layout(int64_t N, int32_t V) {
 
 long long v_pad(int32_t V) { return ceil_div(V, 64) * 64; }
 
+// Backward workspace: [status | count] header, selected-row indices, the
+// gathered hidden rows (zero-padded to 128 rows), then the dZ chunk buffer.
+struct BwdLayout {
+  size_t status_off, count_off, idx_off, hc_off, fixed;
+  long long n_pad;
+};
+
+BwdLayout bwd_layout(int64_t N, int32_t d) {
+  BwdLayout L;
+  L.n_pad = ceil_div(N, kBM) * kBM;
+  L.status_off = 0;
+  L.count_off = 128;
+  L.idx_off = kStatusBytes;
+  L.hc_off = align_up(L.idx_off + size_t(L.n_pad) * 4, 256);
+  L.fixed = align_up(L.hc_off + size_t(L.n_pad) * size_t(d) * 2, 256);
+  return L;
+}
+
 }  // namespace
 
 extern "C" {
@@ -238,14 +256,14 @@ size_t mc_token_logprobs_bwd_workspace_size(int64_t N, int32_t d, int32_t V, int
   if (!valid_common(N, d, V, 1.f) || rows_per_chunk < 1) return 0;
   long long r = rows_per_chunk < N ? rows_per_chunk : N;
   r = ceil_div(r < 1 ? 1 : r, kBM) * kBM;
-  return kStatusBytes + align_up(size_t(r) * size_t(v_pad(V)) * 2, 256);
+  return bwd_layout(N, d).fixed + align_up(size_t(r) * size_t(v_pad(V)) * 2, 256);
 }
 
 mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const int32_t* targets, const float* lse,
-                                const float* entropy, const float* grad_logp, const float* grad_entropy, int64_t N,
-                                int32_t d, int32_t V, float inv_temperature, void* grad_hidden, float* grad_w,
-                                int32_t accumulate, void* workspace, size_t workspace_bytes, int32_t* dev_status,
-                                mc_stream_t stream) {
+                                const float* entropy, const float* grad_logp, const float* grad_entropy,
+                                const uint8_t* row_keep, int64_t N, int32_t d, int32_t V, float inv_temperature,
+                                void* grad_hidden, float* grad_w, int32_t accumulate, void* workspace,
+                                size_t workspace_bytes, int32_t* dev_status, mc_stream_t stream) {
   if (!valid_common(N, d, V, inv_temperature)) return MC_ERR_INVALID_ARG;
   if (!grad_w || !aligned(grad_w, 16)) return MC_ERR_INVALID_ARG;
   if (N > 0) {
@@ -257,14 +275,14 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
       return MC_ERR_INVALID_ARG;
   }
   const long long vp = v_pad(V);
+  const BwdLayout L = bwd_layout(N, d);
   long long R = 0;
   if (N > 0) {
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < mc_token_logprobs_bwd_workspace_size(N, d, V, kBM))
       return MC_ERR_WORKSPACE;
-    R = static_cast<long long>((workspace_bytes - kStatusBytes) / (size_t(vp) * 2));
+    R = static_cast<long long>((workspace_bytes - L.fixed) / (size_t(vp) * 2));
     R = R / kBM * kBM;
-    const long long n_pad = ceil_div(N, kBM) * kBM;
-    if (R > n_pad) R = n_pad;
+    if (R > L.n_pad) R = L.n_pad;
     if (R < kBM) return MC_ERR_WORKSPACE;
   }
   int sms = 0;
@@ -280,30 +298,53 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     return MC_OK;
   }
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  int32_t* ws_status = reinterpret_cast<int32_t*>(ws);
-  void* dz = ws + kStatusBytes;
-  e = cudaMemsetAsync(ws_status, 0, sizeof(int32_t), s);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  int32_t* ws_status = reinterpret_cast<int32_t*>(ws + L.status_off);
+  int32_t* count = reinterpret_cast<int32_t*>(ws + L.count_off);
+  int32_t* idx = reinterpret_cast<int32_t*>(ws + L.idx_off);
+  uint16_t* hc = reinterpret_cast<uint16_t*>(ws + L.hc_off);
+  void* dz = ws + L.fixed;
+  if ((e = cudaMemsetAsync(ws, 0, kStatusBytes, s)) != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  // Rows outside the selection keep a zero gradient.
+  if ((e = cudaMemsetAsync(grad_hidden, 0, size_t(N) * size_t(d) * 2, s)) != cudaSuccess)
+    return cuda_fail(e, "cudaMemsetAsync");
+
+  const uint64_t tmo = wait_timeout_ns();
+  mc::SelectArgs sa;
+  sa.hidden = hidden;
+  sa.row_keep = row_keep;
+  sa.grad_logp = grad_logp;
+  sa.grad_entropy = grad_entropy;
+  sa.targets = targets;
+  sa.N = N;
+  sa.d = d;
+  sa.V = V;
+  sa.idx = idx;
+  sa.count = count;
+  sa.hc = hc;
+  sa.ws_status = ws_status;
+  sa.grid = sms * 8;
+  if ((e = mc::launch_select_gather(sa, s)) != cudaSuccess) return cuda_fail(e, "row selection launch");
 
   CUtensorMap tm_w_k, tm_w_mn;
   if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, kBN)) != MC_OK) return st;
   if ((st = make_tmap(&tm_w_mn, w_vocab, d, V, d, 64)) != MC_OK) return st;
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
-  const uint64_t tmo = wait_timeout_ns();
-  const uint16_t* h16 = static_cast<const uint16_t*>(hidden);
-  uint16_t* gh16 = static_cast<uint16_t*>(grad_hidden);
 
+  // Chunks of R compacted rows; chunks past the device-side count do no work.
   for (long long r0 = 0; r0 < N; r0 += R) {
     const long long rows = (N - r0) < R ? (N - r0) : R;
-    const void* h_chunk = h16 + r0 * d;
+    const void* hc_chunk = hc + r0 * d;
     mc::DzArgs za;
-    if ((st = make_tmap(&za.tm_hidden, h_chunk, d, rows, d, kBM)) != MC_OK) return st;
+    if ((st = make_tmap(&za.tm_hidden, hc_chunk, d, rows, d, kBM)) != MC_OK) return st;
     za.tm_w = tm_w_k;
-    za.targets = targets + r0;
-    za.lse = lse + r0;
-    za.entropy = entropy ? entropy + r0 : nullptr;
-    za.grad_logp = grad_logp + r0;
-    za.grad_entropy = grad_entropy ? grad_entropy + r0 : nullptr;
+    za.targets = targets;
+    za.lse = lse;
+    za.entropy = entropy;
+    za.grad_logp = grad_logp;
+    za.grad_entropy = grad_entropy;
+    za.idx = idx + r0;
+    za.count = count;
+    za.row_offset = r0;
     za.rows = rows;
     za.d = d;
     za.V = V;
@@ -319,10 +360,13 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     mc::DhArgs ha;
     if ((st = make_tmap(&ha.tm_dz, dz, V, rows, vp, kBM)) != MC_OK) return st;
     ha.tm_w_mn = tm_w_mn;
+    ha.idx = idx + r0;
+    ha.count = count;
+    ha.row_offset = r0;
     ha.rows = rows;
     ha.d = d;
     ha.V = V;
-    ha.grad_hidden = gh16 + r0 * d;
+    ha.grad_hidden = grad_hidden;
     ha.ws_status = ws_status;
     ha.grid = sms;
     ha.timeout_ns = tmo;
@@ -330,7 +374,9 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
 
     mc::DwArgs wa;
     if ((st = make_tmap(&wa.tm_dz_mn, dz, V, rows, vp, 64)) != MC_OK) return st;
-    if ((st = make_tmap(&wa.tm_h_mn, h_chunk, d, rows, d, 64)) != MC_OK) return st;
+    if ((st = make_tmap(&wa.tm_h_mn, hc_chunk, d, rows, d, 64)) != MC_OK) return st;
+    wa.count = count;
+    wa.row_offset = r0;
     wa.rows = rows;
     wa.d = d;
     wa.V = V;

@@ -1,13 +1,19 @@
 // mc_bwd.cu — backward of the fused log-prob / entropy forward.
 //
+// Stage 0 (row selection): rows whose effective upstream gradient is zero
+// (row_keep[t] == 0, i.e. M_i = 0 in Eq. 17, or g_t = gH_t = 0, or an invalid
+// target) contribute nothing; one CTA scans the rows in order and writes the
+// indices of the others (idx[], count). Their hidden rows are gathered into a
+// dense block Hc, zero-padded to a multiple of 128 rows. All later extents come
+// from the device-side count, so nothing waits on the host.
 // Stage 1 (dZ producer): the forward's tensor-core mainloop recomputes each
-// 128 x 256 logit tile in TMEM; the epilogue turns it into
+// 128 x 256 logit tile of the selected rows in TMEM; the epilogue turns it into
 //     p        = 2^(z log2e - lse log2e)
-//     dZ[t, v] = inv_temp ( g_t (1[v = y_t] - p) - gH_t p (log p + H_t) )
+//     dZ[j, v] = inv_temp ( g (1[v = y] - p) - gH p (log p + H) )
 // and stores dZ as bf16 (a gradient, not the logits) to the workspace.
-// Stage 2: grad_hidden = dZ . W     (A = dZ K-major, B = W read N-major)
-// Stage 3: grad_w (+)= dZ^T . H     (A = dZ read M-major, B = H read N-major)
-// Both are plain tcgen05 GEMMs of the same engine with store epilogues.
+// Stage 2: grad_hidden[idx[j]] = (dZ . W)[j]   (A = dZ K-major, B = W N-major)
+// Stage 3: grad_w (+)= dZ^T . Hc                (A = dZ M-major, B = Hc N-major)
+// Stages 2-3 are plain tcgen05 GEMMs of the same engine with store epilogues.
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
@@ -19,11 +25,78 @@ namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kSelectThreads = 1024;
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&v);
 }
+
+// ---------------------------------------------------------------- stage 0
+
+// One CTA: ordered compaction of the rows with a nonzero effective upstream
+// gradient. Block-wide exclusive scan per 1024-row slab (warp ballots, then a
+// warp scan of the 32 warp counts).
+__global__ void __launch_bounds__(kSelectThreads) select_rows_kernel(
+    const uint8_t* __restrict__ row_keep, const float* __restrict__ g, const float* __restrict__ gh,
+    const int32_t* __restrict__ targets, int V, long long N, int32_t* __restrict__ idx, int32_t* count,
+    int32_t* status) {
+  __shared__ int warp_off[kSelectThreads / 32];
+  __shared__ int slab_total;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int base = 0;
+  bool bad_target = false;
+  for (long long start = 0; start < N; start += kSelectThreads) {
+    const long long t = start + tid;
+    int f = 0;
+    if (t < N) {
+      const int y = targets[t];
+      const bool yok = y >= 0 && y < V;
+      bad_target |= !yok;
+      const bool live = g[t] != 0.f || (gh != nullptr && gh[t] != 0.f);
+      f = (yok && live && (row_keep == nullptr || row_keep[t] != 0)) ? 1 : 0;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, f);
+    const int in_warp = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) warp_off[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+      const int c = warp_off[lane];
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      warp_off[lane] = incl - c;
+      if (lane == 31) slab_total = incl;
+    }
+    __syncthreads();
+    if (f) idx[base + warp_off[warp] + in_warp] = static_cast<int32_t>(t);
+    base += slab_total;
+    __syncthreads();
+  }
+  if (__syncthreads_or(bad_target) && tid == 0) atomicOr(status, MC_DEV_TARGET_RANGE);
+  if (tid == 0) *count = base;
+}
+
+// Hc[j] = H[idx[j]] for j < count, zero rows up to the next multiple of 128.
+__global__ void gather_rows_kernel(const uint4* __restrict__ H, int row_vec, const int32_t* __restrict__ idx,
+                                   const int32_t* __restrict__ count, uint4* __restrict__ Hc) {
+  const long long cnt = *count;
+  const long long lim = (cnt + BM - 1) / BM * BM;
+  for (long long j = blockIdx.x; j < lim; j += gridDim.x) {
+    uint4* dst = Hc + j * row_vec;
+    if (j < cnt) {
+      const uint4* src = H + static_cast<long long>(idx[j]) * row_vec;
+      for (int k = threadIdx.x; k < row_vec; k += blockDim.x) dst[k] = src[k];
+    } else {
+      for (int k = threadIdx.x; k < row_vec; k += blockDim.x) dst[k] = make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+
+// ---------------------------------------------------------------- stage 1
 
 struct DzEpi {
   struct Params {
@@ -32,36 +105,39 @@ struct DzEpi {
     const float* entropy;
     const float* grad_logp;
     const float* grad_entropy;
-    long long rows;
+    const int32_t* idx;  // compacted row -> original row (this chunk's slice)
+    long long rows;      // rows of this chunk (host bound; the device count may be lower)
     int V;
     float scale2;
     float inv_temp;
     __nv_bfloat16* dz;
     long long ld;
-    int32_t* status;
   };
 
+  long long rows_lim;
   float lse2, cg, cgh, hrow;
   int y;
   bool valid;
 
+  __device__ __forceinline__ void setup(const Params& p, long long rows_eff, bool) {
+    rows_lim = rows_eff >= 0 ? rows_eff : p.rows;
+  }
+
   __device__ __forceinline__ void begin(const Params& p, long long row, int, int) {
-    valid = row < p.rows;
+    valid = row < rows_lim;
     y = -1;
     lse2 = cg = cgh = hrow = 0.f;
     if (!valid) return;
-    y = __ldg(p.targets + row);
-    cg = __ldg(p.grad_logp + row) * p.inv_temp;
-    cgh = p.grad_entropy ? __ldg(p.grad_entropy + row) * p.inv_temp : 0.f;
-    hrow = (p.grad_entropy && p.entropy) ? __ldg(p.entropy + row) : 0.f;
-    lse2 = __ldg(p.lse + row) * kLog2e;
-    if (y < 0 || y >= p.V) {  // invalid target: drop the row's gradient terms
-      atomicOr(p.status, MC_DEV_TARGET_RANGE);
-      cg = cgh = 0.f;
-      lse2 = 0.f;
-    }
+    const long long o = p.idx ? p.idx[row] : row;
+    y = __ldg(p.targets + o);
+    cg = __ldg(p.grad_logp + o) * p.inv_temp;
+    cgh = p.grad_entropy ? __ldg(p.grad_entropy + o) * p.inv_temp : 0.f;
+    hrow = (p.grad_entropy && p.entropy) ? __ldg(p.entropy + o) : 0.f;
+    lse2 = __ldg(p.lse + o) * kLog2e;
   }
 
+  // Rows past the device count inside the last row block get dZ = 0, so the
+  // K tail of the grad_w GEMM reads zeros.
   __device__ __forceinline__ void tile(const Params& p, long long row, int n_tile, uint32_t taddr) {
     const int v0 = n_tile * BN;
 #pragma unroll 1
@@ -69,20 +145,25 @@ struct DzEpi {
       float x[32];
       tmem_ld32(taddr + c * 32, x);
       const int vc = v0 + c * 32;
-      if (!valid || vc >= p.V) continue;
-      const float nl = -lse2;
+      if (vc >= p.V || row >= p.rows) continue;
       uint32_t w[16];
+      if (valid) {
+        const float nl = -lse2;
 #pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        float d2[2];
+        for (int i = 0; i < 32; i += 2) {
+          float d2[2];
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          const float a = fmaf(x[i + j], p.scale2, nl);  // log2 p
-          const float pr = ex2_approx(a);
-          const float oh = (vc + i + j == y) ? 1.f : 0.f;
-          d2[j] = fmaf(cg, oh - pr, -cgh * pr * fmaf(a, kLn2, hrow));
+          for (int j = 0; j < 2; ++j) {
+            const float a = fmaf(x[i + j], p.scale2, nl);  // log2 p
+            const float pr = ex2_approx(a);
+            const float oh = (vc + i + j == y) ? 1.f : 0.f;
+            d2[j] = fmaf(cg, oh - pr, -cgh * pr * fmaf(a, kLn2, hrow));
+          }
+          w[i / 2] = pack_bf16x2(d2[0], d2[1]);
         }
-        w[i / 2] = pack_bf16x2(d2[0], d2[1]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) w[i] = 0u;
       }
       __nv_bfloat16* dst = p.dz + row * p.ld + vc;
       if (vc + 32 <= p.V) {
@@ -91,11 +172,10 @@ struct DzEpi {
         for (int q = 0; q < 4; ++q) d4[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
       } else {
         const int n = p.V - vc;
-        for (int i = 0; i < n; ++i) {
-          const uint32_t pair = w[i / 2];
-          const uint16_t bits = (i & 1) ? static_cast<uint16_t>(pair >> 16) : static_cast<uint16_t>(pair & 0xFFFFu);
-          reinterpret_cast<uint16_t*>(dst)[i] = bits;
-        }
+        uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (i < n) d16[i] = static_cast<uint16_t>((i & 1) ? (w[i / 2] >> 16) : (w[i / 2] & 0xFFFFu));
       }
     }
   }
@@ -103,24 +183,32 @@ struct DzEpi {
   __device__ __forceinline__ void end(const Params&, long long, int, int, bool) {}
 };
 
-// out[row, col] = acc (bf16), rows < p.rows, cols < p.cols (cols % 32 == 0).
+// ---------------------------------------------------------------- stages 2-3
+
+// out[idx[row], col] = acc (bf16) for row < rows (device count), col < cols (cols % 32 == 0).
 struct StoreBf16Epi {
   struct Params {
     __nv_bfloat16* out;
+    const int32_t* idx;  // nullable: identity
     long long ld;
     long long rows;
     int cols;
   };
+  long long rows_lim;
+  __device__ __forceinline__ void setup(const Params& p, long long rows_eff, bool) {
+    rows_lim = rows_eff >= 0 ? rows_eff : p.rows;
+  }
   __device__ __forceinline__ void begin(const Params&, long long, int, int) {}
   __device__ __forceinline__ void tile(const Params& p, long long row, int n_tile, uint32_t taddr) {
     const int n0 = n_tile * BN;
+    const long long orow = (row < rows_lim) ? (p.idx ? p.idx[row] : row) : -1;
 #pragma unroll 1
     for (int c = 0; c < BN / 32; ++c) {
       float x[32];
       tmem_ld32(taddr + c * 32, x);
       const int col = n0 + c * 32;
-      if (row >= p.rows || col >= p.cols) continue;
-      uint4* d4 = reinterpret_cast<uint4*>(p.out + row * p.ld + col);
+      if (orow < 0 || col >= p.cols) continue;
+      uint4* d4 = reinterpret_cast<uint4*>(p.out + orow * p.ld + col);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
         d4[q] = make_uint4(pack_bf16x2(x[8 * q + 0], x[8 * q + 1]), pack_bf16x2(x[8 * q + 2], x[8 * q + 3]),
@@ -131,6 +219,8 @@ struct StoreBf16Epi {
 };
 
 // out[row, col] (+)= acc (fp32), rows < p.rows, cols < p.cols (cols % 32 == 0).
+// With an empty K extent the product is zero: overwrite writes zeros,
+// accumulate leaves `out` as it is.
 struct StoreF32Epi {
   struct Params {
     float* out;
@@ -139,6 +229,8 @@ struct StoreF32Epi {
     int cols;
     int accumulate;
   };
+  bool kvalid;
+  __device__ __forceinline__ void setup(const Params&, long long, bool k_nonempty) { kvalid = k_nonempty; }
   __device__ __forceinline__ void begin(const Params&, long long, int, int) {}
   __device__ __forceinline__ void tile(const Params& p, long long row, int n_tile, uint32_t taddr) {
     const int n0 = n_tile * BN;
@@ -148,10 +240,12 @@ struct StoreF32Epi {
       tmem_ld32(taddr + c * 32, x);
       const int col = n0 + c * 32;
       if (row >= p.rows || col >= p.cols) continue;
+      if (!kvalid && p.accumulate) continue;
       float4* d4 = reinterpret_cast<float4*>(p.out + row * p.ld + col);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
-        float4 v = make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3]);
+        float4 v = kvalid ? make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3])
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
         if (p.accumulate) {
           const float4 o = d4[q];
           v.x += o.x;
@@ -174,7 +268,7 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(GEMM_SMEM_BYTES));
   if (e != cudaSuccess) return e;
-  const int units = sch.m_blocks * sch.splits;
+  const int units = sch.m_blocks * sch.splits;  // host upper bound; the kernel may find fewer
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
   kern<<<grid, GEMM_THREADS, GEMM_SMEM_BYTES, stream>>>(ta, tb, sch, ep, timeout_ns, status);
@@ -187,25 +281,40 @@ __global__ void status_merge(const int32_t* ws_status, int32_t* dev_status) {
 
 }  // namespace
 
+cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
+  select_rows_kernel<<<1, kSelectThreads, 0, stream>>>(a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V,
+                                                       a.N, a.idx, a.count, a.ws_status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int row_vec = a.d * 2 / 16;
+  gather_rows_kernel<<<a.grid, 256, 0, stream>>>(static_cast<const uint4*>(a.hidden), row_vec, a.idx, a.count,
+                                                 static_cast<uint4*>(a.hc));
+  return cudaGetLastError();
+}
+
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   Schedule sch;
   sch.m_blocks = static_cast<int>((a.rows + BM - 1) / BM);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
   sch.k_blocks = a.d / BK;
+  sch.dyn_count = a.count;
+  sch.dyn_offset = a.row_offset;
+  sch.dyn_cap = a.rows;
+  sch.dyn_mode = DYN_ROWS;
   DzEpi::Params ep;
   ep.targets = a.targets;
   ep.lse = a.lse;
   ep.entropy = a.entropy;
   ep.grad_logp = a.grad_logp;
   ep.grad_entropy = a.grad_entropy;
+  ep.idx = a.idx;
   ep.rows = a.rows;
   ep.V = a.V;
   ep.scale2 = a.inv_temperature * kLog2e;
   ep.inv_temp = a.inv_temperature;
   ep.dz = static_cast<__nv_bfloat16*>(a.dz);
   ep.ld = a.ld;
-  ep.status = a.ws_status;
   return run_gemm<DzEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
                                        stream);
 }
@@ -216,8 +325,13 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;  // one output tile per unit
   sch.k_blocks = (a.V + BK - 1) / BK;
+  sch.dyn_count = a.count;
+  sch.dyn_offset = a.row_offset;
+  sch.dyn_cap = a.rows;
+  sch.dyn_mode = DYN_ROWS;
   StoreBf16Epi::Params ep;
   ep.out = static_cast<__nv_bfloat16*>(a.grad_hidden);
+  ep.idx = a.idx;
   ep.ld = a.d;
   ep.rows = a.rows;
   ep.cols = a.d;
@@ -231,6 +345,10 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;
   sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);
+  sch.dyn_count = a.count;
+  sch.dyn_offset = a.row_offset;
+  sch.dyn_cap = a.rows;
+  sch.dyn_mode = DYN_K;
   StoreF32Epi::Params ep;
   ep.out = a.grad_w;
   ep.ld = a.d;

@@ -41,6 +41,8 @@ struct FwdEpi {
   float m, s0, s1, t0, t1;
   int y;
 
+  __device__ __forceinline__ void setup(const Params&, long long, bool) {}
+
   __device__ __forceinline__ void begin(const Params& p, long long row, int, int) {
     m = -INFINITY;
     s0 = s1 = t0 = t1 = 0.f;

@@ -66,11 +66,20 @@ struct GemmShared {
 
 constexpr size_t GEMM_SMEM_BYTES = size_t(NUM_STAGES) * STAGE_BYTES + sizeof(GemmShared) + 1024;
 
+enum DynMode : int { DYN_NONE = 0, DYN_ROWS = 1, DYN_K = 2 };
+
 struct Schedule {
   int m_blocks;  // ceil(M / BM)
   int n_tiles;   // ceil(N / BN)
   int splits;    // tile ranges per row block, 1 <= splits <= n_tiles
   int k_blocks;  // ceil(K / BK)
+  // Optional extent known only on the device (a count written by an earlier
+  // kernel on the stream): c = clamp(*dyn_count - dyn_offset, 0, dyn_cap)
+  // replaces M (DYN_ROWS: m_blocks = ceil(c / BM)) or K (DYN_K).
+  const int32_t* dyn_count = nullptr;
+  long long dyn_offset = 0;
+  long long dyn_cap = 0;
+  int dyn_mode = DYN_NONE;
 
   __device__ __forceinline__ int units() const { return m_blocks * splits; }
   __device__ __forceinline__ void unit(int u, int& mb, int& split, int& t0, int& t1) const {
@@ -84,6 +93,7 @@ struct Schedule {
 // Epilogue functor contract (one instance per epilogue thread):
 //   struct Epi {
 //     struct Params;
+//     __device__ void setup(const Params&, long long rows_eff, bool k_nonempty);
 //     __device__ void begin(const Params&, long long row, int mb, int split);
 //     __device__ void tile(const Params&, long long row, int n_tile, uint32_t taddr);
 //     __device__ void end(const Params&, long long row, int mb, int split, bool ok);
@@ -91,12 +101,29 @@ struct Schedule {
 // `row` = global M index of the thread's row (may be >= M: padding rows),
 // `taddr` = TMEM address of the thread's warp's lane quadrant, column 0 of the
 // accumulator holding tile `n_tile`. `ok` is false when the pipeline gave up.
+// `rows_eff` is the device-side row count under DYN_ROWS (else -1);
+// `k_nonempty` is false when a DYN_K extent is 0 (the accumulator is then
+// never written and must be read as zero).
 
 template <class Epi, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const Schedule sch, const typename Epi::Params ep, const uint64_t timeout_ns,
+                    const Schedule sch_in, const typename Epi::Params ep, const uint64_t timeout_ns,
                     int32_t* dev_status) {
+  Schedule sch = sch_in;
+  long long rows_eff = -1;
+  bool k_nonempty = true;
+  if (sch.dyn_count != nullptr) {
+    long long c = static_cast<long long>(*sch.dyn_count) - sch.dyn_offset;
+    c = c < 0 ? 0 : (c > sch.dyn_cap ? sch.dyn_cap : c);
+    if (sch.dyn_mode == DYN_ROWS) {
+      sch.m_blocks = static_cast<int>((c + BM - 1) / BM);
+      rows_eff = c;
+    } else if (sch.dyn_mode == DYN_K) {
+      sch.k_blocks = static_cast<int>((c + BK - 1) / BK);
+      k_nonempty = sch.k_blocks > 0;
+    }
+  }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   GemmShared* sh = reinterpret_cast<GemmShared*>(smem + NUM_STAGES * STAGE_BYTES);
@@ -228,6 +255,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t tc = 0;
     Epi epi;
+    epi.setup(ep, rows_eff, k_nonempty);
     bool ok = true;
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       int mb, split, t0, t1;

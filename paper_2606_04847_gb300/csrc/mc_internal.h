@@ -32,16 +32,36 @@ struct FwdArgs {
 };
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream);
 
-// Backward building blocks.
-struct DzArgs {
-  CUtensorMap tm_hidden;  // K-major {d, rows}, box {64, 128}
-  CUtensorMap tm_w;       // K-major {d, V}, box {64, 256}
+// Backward building blocks. Rows are first compacted on the device (idx[],
+// *count); every later stage takes its extent from *count.
+struct SelectArgs {
+  const void* hidden;     // bf16 [N, d]
+  const uint8_t* row_keep;
+  const float* grad_logp;
+  const float* grad_entropy;
   const int32_t* targets;
+  long long N;
+  int d, V;
+  int32_t* idx;           // workspace: [N] selected original rows, ascending
+  int32_t* count;         // workspace: number selected
+  void* hc;               // workspace: bf16 [n_pad, d] gathered hidden rows
+  int32_t* ws_status;
+  int grid;
+};
+cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream);
+
+struct DzArgs {
+  CUtensorMap tm_hidden;  // K-major {d, rows} over Hc + row_offset, box {64, 128}
+  CUtensorMap tm_w;       // K-major {d, V}, box {64, 256}
+  const int32_t* targets; // original-row arrays (indexed through idx)
   const float* lse;
   const float* entropy;
   const float* grad_logp;
   const float* grad_entropy;
-  long long rows;
+  const int32_t* idx;     // idx + row_offset
+  const int32_t* count;
+  long long row_offset;   // first compacted row of this chunk
+  long long rows;         // chunk capacity (rows of the dZ buffer used)
   int d, V;
   float inv_temperature;
   int splits;
@@ -53,21 +73,26 @@ struct DzArgs {
 };
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream);
 
-struct DhArgs {           // grad_hidden[rows, d] = dZ[rows, V] . W[V, d]
+struct DhArgs {           // grad_hidden[idx[j], :] = (dZ . W)[j, :]
   CUtensorMap tm_dz;      // K-major {V, rows}, box {64, 128}
   CUtensorMap tm_w_mn;    // N-major {d, V}, box {64, 64}
+  const int32_t* idx;     // idx + row_offset
+  const int32_t* count;
+  long long row_offset;
   long long rows;
   int d, V;
-  void* grad_hidden;      // bf16, row stride d
+  void* grad_hidden;      // bf16 [N, d]
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
 };
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream);
 
-struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . H[rows, d]
+struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . Hc[rows, d]
   CUtensorMap tm_dz_mn;   // M-major {V, rows}, box {64, 64}
-  CUtensorMap tm_h_mn;    // N-major {d, rows}, box {64, 64}
+  CUtensorMap tm_h_mn;    // N-major {d, rows} over Hc + row_offset, box {64, 64}
+  const int32_t* count;
+  long long row_offset;
   long long rows;
   int d, V;
   float* grad_w;

@@ -44,8 +44,8 @@ SIGNATURES = {
     "mc_token_logprobs_workspace_size": (_SZ, [_I64, _I32, _I32]),
     "mc_token_logprobs": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _SZ, _P, _P]),
     "mc_token_logprobs_bwd_workspace_size": (_SZ, [_I64, _I32, _I32, _I64]),
-    "mc_token_logprobs_bwd": (_I32, [_P, _P, _P, _P, _P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _I32, _P, _SZ,
-                                     _P, _P]),
+    "mc_token_logprobs_bwd": (_I32, [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _I32, _P,
+                                     _SZ, _P, _P]),
     "mc_seq_ratio_filter": (_I32, [_P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _P, _P, _P]),
     "mc_selftest_bounded_wait": (_I32, [_P, _I64, _P]),
 }
@@ -146,6 +146,7 @@ def token_logprobs(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.T
 def token_logprobs_bwd(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.Tensor, lse: torch.Tensor,
                        entropy: Optional[torch.Tensor], grad_logp: torch.Tensor,
                        grad_entropy: Optional[torch.Tensor] = None, inv_temperature: float = 1.0, *,
+                       row_keep: Optional[torch.Tensor] = None,
                        grad_hidden: Optional[torch.Tensor] = None, grad_w: Optional[torch.Tensor] = None,
                        accumulate: bool = False, workspace: Optional[torch.Tensor] = None,
                        rows_per_chunk: Optional[int] = None, dev_status: Optional[torch.Tensor] = None,
@@ -156,6 +157,8 @@ def token_logprobs_bwd(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: tor
     _need(targets, "targets", torch.int32, 1)
     _need(lse, "lse", torch.float32, 1)
     _need(grad_logp, "grad_logp", torch.float32, 1)
+    if row_keep is not None:
+        _need(row_keep, "row_keep", torch.uint8, 1)
     N, d = hidden.shape
     V = w_vocab.shape[0]
     dev = hidden.device
@@ -167,7 +170,8 @@ def token_logprobs_bwd(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: tor
         need = backward_workspace_size(N, d, V, rows_per_chunk)
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
     st = lib().mc_token_logprobs_bwd(_ptr(hidden), _ptr(w_vocab), _ptr(targets), _ptr(lse), _ptr(entropy),
-                                     _ptr(grad_logp), _ptr(grad_entropy), N, d, V, float(inv_temperature),
+                                     _ptr(grad_logp), _ptr(grad_entropy), _ptr(row_keep), N, d, V,
+                                     float(inv_temperature),
                                      _ptr(grad_hidden), _ptr(grad_w), int(bool(accumulate)), _ptr(workspace),
                                      workspace.numel(), _ptr(dev_status), _stream(stream))
     _check("mc_token_logprobs_bwd", st)

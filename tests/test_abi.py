@@ -98,7 +98,7 @@ def test_forward_without_gpu_reports_device_error(L):
 
 
 def bwd(L, N=256, d=512, V=4096, ws_bytes=1 << 30, grad_w=FAKE, grad_entropy=None, entropy=None):
-    return L.mc_token_logprobs_bwd(FAKE, FAKE, FAKE, FAKE, entropy, FAKE, grad_entropy, N, d, V, 1.0, FAKE,
+    return L.mc_token_logprobs_bwd(FAKE, FAKE, FAKE, FAKE, entropy, FAKE, grad_entropy, None, N, d, V, 1.0, FAKE,
                                    grad_w, 0, FAKE, ws_bytes, None, None)
 
 

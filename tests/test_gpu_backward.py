@@ -87,3 +87,20 @@ def test_vocab_tail_and_large_hidden():
 
 def test_peaked_softmax():
     check(*setup(256, 256, 2048, seed=6, w_scale=8.0))
+
+
+def test_row_keep_gate_equals_zeroed_upstream():
+    """row_keep = 0 on a dropped sequence gives the same gradients as zeroing
+    its upstream gradient (the M_i factor of Eq. 17)."""
+    wl, g, ge = setup(384, 128, 1500, seed=7)
+    keep = torch.ones(384, dtype=torch.uint8)
+    keep[100:260] = 0
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    fw = mc.token_logprobs(h, w, y)
+    a = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda(), row_keep=keep.cuda())
+    g0, ge0 = g * keep.float(), ge * keep.float()
+    b = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g0.cuda(), ge0.cuda())
+    assert torch.equal(a["grad_hidden"], b["grad_hidden"])
+    assert torch.equal(a["grad_w"], b["grad_w"])
+    ref = oracle.token_logprobs_bwd(wl.hidden, wl.w_vocab, wl.targets, g0, ge0)
+    assert rel_fro(np_(a["grad_w"]), ref["grad_w"]) <= TOL_GRAD
