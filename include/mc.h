@@ -47,7 +47,9 @@ typedef enum {
   MC_ERR_CUDA = 3,          /* a CUDA runtime or driver call failed; see mc_last_cuda_error() */
   MC_ERR_TIMEOUT = 4,       /* reported through dev_status: see MC_DEV_TIMEOUT */
   MC_ERR_WORKSPACE = 5,     /* workspace pointer null/misaligned or smaller than the query */
-  MC_ERR_TARGET_RANGE = 6   /* reported through dev_status: see MC_DEV_TARGET_RANGE */
+  MC_ERR_TARGET_RANGE = 6,  /* reported through dev_status: see MC_DEV_TARGET_RANGE */
+  MC_ERR_SCRATCH_LIMIT = 7  /* mc_token_logprobs_noalloc: the request needs more scratch than
+                               the library's fixed MC_NOALLOC_SCRATCH_BYTES */
 } mc_status;
 
 /* Bits the kernels OR into *dev_status (an int32 in device memory). */
@@ -94,6 +96,37 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
                             float* logp, float* entropy, float* lse,
                             void* workspace, size_t workspace_bytes,
                             int32_t* dev_status, mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Forward for callers that cannot allocate device memory. (The paper has no
+ * counterpart: this is a deployment variant of mc_token_logprobs.)
+ *
+ * Some callers may not call cudaMalloc and have no spare buffer to pass as a
+ * workspace: a host process whose memory manager owns every device
+ * allocation, a plugin running inside such a host, or a latency-critical loop
+ * that cannot take the device-wide synchronisation an allocation may cause.
+ * This entry point computes exactly what mc_token_logprobs computes, with the
+ * same arguments minus the workspace; its scratch is a fixed array of
+ * MC_NOALLOC_SCRATCH_BYTES compiled into libmc, which every GPU that loads
+ * the library holds until the process exits. It allocates nothing itself.
+ *
+ *   Limit: requests with mc_token_logprobs_workspace_size(N, d, V) greater than
+ *   MC_NOALLOC_SCRATCH_BYTES are rejected with MC_ERR_SCRATCH_LIMIT before any
+ *   work is queued (about 171,000 rows for V >= 4096; more for smaller V).
+ *   Set-up: the first call on each device looks up the array's device address
+ *   with that device current and caches it; make that first call before any
+ *   stream capture begins.
+ *   Sharing: all calls on a device use the same array and it keeps the last
+ *   call's contents (the call clears, on its stream, what must start at zero).
+ *   Calls whose work overlaps on the GPU (different streams without ordering
+ *   between them) race on the array; order them.
+ * ------------------------------------------------------------------------ */
+#define MC_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+mc_status mc_token_logprobs_noalloc(const void* hidden, const void* w_vocab, const int32_t* targets,
+                                    int64_t N, int32_t d, int32_t V, float inv_temperature,
+                                    float* logp, float* entropy, float* lse,
+                                    int32_t* dev_status, mc_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * Backward of the forward above.

@@ -193,6 +193,8 @@ const char* mc_status_string(mc_status s) {
     case MC_ERR_TIMEOUT: return "MC_ERR_TIMEOUT: a bounded device wait gave up";
     case MC_ERR_WORKSPACE: return "MC_ERR_WORKSPACE: workspace missing, misaligned or too small";
     case MC_ERR_TARGET_RANGE: return "MC_ERR_TARGET_RANGE: a target index outside [0, V)";
+    case MC_ERR_SCRATCH_LIMIT:
+      return "MC_ERR_SCRATCH_LIMIT: request needs more than the fixed MC_NOALLOC_SCRATCH_BYTES scratch";
   }
   return "unknown mc_status";
 }

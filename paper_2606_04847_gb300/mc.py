@@ -27,6 +27,7 @@ STATUS_NAMES = {
     4: "MC_ERR_TIMEOUT",
     5: "MC_ERR_WORKSPACE",
     6: "MC_ERR_TARGET_RANGE",
+    7: "MC_ERR_SCRATCH_LIMIT",
 }
 MC_DEV_TIMEOUT = 0x1
 MC_DEV_TARGET_RANGE = 0x2
@@ -43,6 +44,7 @@ SIGNATURES = {
     "mc_version": (_I32, []),
     "mc_token_logprobs_workspace_size": (_SZ, [_I64, _I32, _I32]),
     "mc_token_logprobs": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _SZ, _P, _P]),
+    "mc_token_logprobs_noalloc": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _P]),
     "mc_token_logprobs_bwd_workspace_size": (_SZ, [_I64, _I32, _I32, _I64]),
     "mc_token_logprobs_bwd": (_I32, [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _I32, _P,
                                      _SZ, _P, _P]),
@@ -140,6 +142,28 @@ def token_logprobs(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.T
                                  _ptr(out["logp"]), _ptr(out.get("entropy")), _ptr(out.get("lse")),
                                  _ptr(workspace), workspace.numel(), _ptr(dev_status), _stream(stream))
     _check("mc_token_logprobs", st)
+    return out
+
+
+def token_logprobs_noalloc(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.Tensor,
+                           inv_temperature: float = 1.0, *, out: dict, dev_status: Optional[torch.Tensor] = None,
+                           stream=None) -> dict:
+    """mc_token_logprobs_noalloc: the forward with the library's fixed scratch.
+
+    For callers that must not allocate device memory: the caller supplies the
+    output tensors in ``out`` ("logp", optional "entropy"/"lse") and nothing is
+    allocated here or in the library. Raises McError(MC_ERR_SCRATCH_LIMIT) when
+    the problem needs more than the fixed scratch.
+    """
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_vocab, "w_vocab", torch.bfloat16, 2)
+    _need(targets, "targets", torch.int32, 1)
+    N, d = hidden.shape
+    V = w_vocab.shape[0]
+    st = lib().mc_token_logprobs_noalloc(_ptr(hidden), _ptr(w_vocab), _ptr(targets), N, d, V,
+                                         float(inv_temperature), _ptr(out["logp"]), _ptr(out.get("entropy")),
+                                         _ptr(out.get("lse")), _ptr(dev_status), _stream(stream))
+    _check("mc_token_logprobs_noalloc", st)
     return out
 
 
