@@ -390,8 +390,8 @@ def run_case(args):
             mc.token_logprobs(h, w, y, out=fw)
         elif args.case == "filter":
             mc.seq_ratio_filter(fw["logp"], lb, None, cu, spec.delta, spec.delta)
-        else:
-            mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], adv, None, row_keep=flt["token_keep"])
+        else:  # every row live, so the capture does not depend on whether the filter keeps this slice
+            mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], adv, None)
     torch.cuda.synchronize()
     print(json.dumps({"case": args.case, "rows": R, "launches": args.launches,
                       "wall_ms_per_launch": (time.perf_counter() - t0) * 1e3 / args.launches}))
