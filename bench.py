@@ -57,7 +57,7 @@ def _peaks():
 
 def _kernel_source_hash():
     h = hashlib.sha256()
-    for f in ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu"):
+    for f in ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu", "mc_api.cu"):
         h.update(open(os.path.join(ROOT, "paper_2606_04847_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 

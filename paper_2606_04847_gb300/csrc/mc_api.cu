@@ -20,8 +20,9 @@
 
 namespace {
 
-constexpr int kBM = 128;
-constexpr int kBN = 256;
+constexpr int kBM = 128;       // rows one CTA owns in a tile (TMA box height for A)
+constexpr int kBN = 256;       // vocabulary / output columns per tile
+constexpr int kRowPad = 256;   // row padding of workspaces: one row block of either engine
 constexpr int kMaxSplits = 16;
 constexpr size_t kStatusBytes = 256;
 constexpr int kMaxDevices = 64;
@@ -77,6 +78,24 @@ uint64_t wait_timeout_ns() {
   return t;
 }
 
+// The one-CTA engine unless MC_ENGINE=pair selects the CTA-pair engine
+// (tcgen05 cta_group::2). Both give the same results; under the GB300's power
+// cap the one-CTA engine sustains a ~10 % higher SM clock and is ~4 % faster
+// on the 9B-class forward, so it is the default.
+bool use_pair_engine() {
+  static const bool pair = [] {
+    const char* s = std::getenv("MC_ENGINE");
+    return s != nullptr && std::strcmp(s, "pair") == 0;
+  }();
+  return pair;
+}
+
+// Rows per scheduled row block, TMA box height of K-major B, and how many
+// units run at once, for the selected engine.
+int row_block() { return use_pair_engine() ? 256 : kBM; }
+int b_box_rows() { return use_pair_engine() ? 128 : kBN; }
+int concurrent_units(int sms) { return use_pair_engine() ? sms / 2 : sms; }
+
 // ---- TMA descriptors
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                               const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -122,13 +141,27 @@ mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
 
 // Vocabulary tile ranges per 128-row block. Enough units to spread over the
 // SMs for small N, and at least 8 so the CTAs running together share few row
-// blocks (their hidden rows stay in L2) for large N.
+// blocks (their hidden rows stay in L2) for large N. Within that range, the
+// count whose units leave the fewest CTAs idle in the last wave (ties: fewer
+// splits, so W is streamed fewer times).
 int choose_splits(long long m_blocks, int n_tiles, int sms) {
-  long long s = ceil_div(2LL * sms, m_blocks);
-  if (s < 8) s = 8;
-  if (s > kMaxSplits) s = kMaxSplits;
-  if (s > n_tiles) s = n_tiles;
-  return static_cast<int>(s < 1 ? 1 : s);
+  long long lo = ceil_div(2LL * sms, m_blocks);
+  if (lo < 8) lo = 8;
+  long long hi = kMaxSplits;
+  if (hi > n_tiles) hi = n_tiles;
+  if (lo > hi) lo = hi;
+  long long best = lo;
+  double best_idle = 2.0;
+  for (long long s = lo; s <= hi; ++s) {
+    const long long units = m_blocks * s;
+    const long long slots = ceil_div(units, sms) * sms;
+    const double idle = static_cast<double>(slots - units) / static_cast<double>(slots);
+    if (idle < best_idle - 1e-9) {
+      best_idle = idle;
+      best = s;
+    }
+  }
+  return static_cast<int>(best < 1 ? 1 : best);
 }
 
 int max_splits(int V) {
@@ -151,7 +184,7 @@ struct FwdLayout {
 
 FwdLayout fwd_layout(int64_t N, int32_t V) {
   FwdLayout L;
-  L.n_pad = ceil_div(N, kBM) * kBM;
+  L.n_pad = ceil_div(N, kRowPad) * kRowPad;
   const size_t part_bytes = size_t(3) * max_splits(V) * size_t(L.n_pad) * 4;
   L.status_off = 0;
   L.part_off = kStatusBytes;
@@ -171,7 +204,7 @@ struct BwdLayout {
 
 BwdLayout bwd_layout(int64_t N, int32_t d) {
   BwdLayout L;
-  L.n_pad = ceil_div(N, kBM) * kBM;
+  L.n_pad = ceil_div(N, kRowPad) * kRowPad;
   L.status_off = 0;
   L.count_off = 128;
   L.idx_off = kStatusBytes;
@@ -228,15 +261,15 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   mc::FwdArgs a;
   if ((st = make_tmap(&a.tm_hidden, hidden, d, N, d, kBM)) != MC_OK) return st;
-  if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, kBN)) != MC_OK) return st;
-  const long long m_blocks = ceil_div(N, kBM);
+  if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, b_box_rows())) != MC_OK) return st;
+  const long long m_blocks = ceil_div(N, row_block());
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
   a.targets = targets;
   a.N = N;
   a.d = d;
   a.V = V;
   a.inv_temperature = inv_temperature;
-  a.splits = choose_splits(m_blocks, n_tiles, sms);
+  a.splits = choose_splits(m_blocks, n_tiles, concurrent_units(sms));
   a.n_pad = L.n_pad;
   a.part = reinterpret_cast<float*>(ws + L.part_off);
   a.zy = reinterpret_cast<float*>(ws + L.zy_off);
@@ -247,6 +280,7 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
   a.dev_status = dev_status;
   a.grid = sms;
   a.timeout_ns = wait_timeout_ns();
+  a.pair = use_pair_engine() ? 1 : 0;
   cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   e = mc::launch_forward(a, s);
@@ -257,7 +291,7 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
 size_t mc_token_logprobs_bwd_workspace_size(int64_t N, int32_t d, int32_t V, int64_t rows_per_chunk) {
   if (!valid_common(N, d, V, 1.f) || rows_per_chunk < 1) return 0;
   long long r = rows_per_chunk < N ? rows_per_chunk : N;
-  r = ceil_div(r < 1 ? 1 : r, kBM) * kBM;
+  r = ceil_div(r < 1 ? 1 : r, kRowPad) * kRowPad;
   return bwd_layout(N, d).fixed + align_up(size_t(r) * size_t(v_pad(V)) * 2, 256);
 }
 
@@ -280,12 +314,12 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
   const BwdLayout L = bwd_layout(N, d);
   long long R = 0;
   if (N > 0) {
-    if (!workspace || !aligned(workspace, 256) || workspace_bytes < mc_token_logprobs_bwd_workspace_size(N, d, V, kBM))
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < mc_token_logprobs_bwd_workspace_size(N, d, V, kRowPad))
       return MC_ERR_WORKSPACE;
     R = static_cast<long long>((workspace_bytes - L.fixed) / (size_t(vp) * 2));
-    R = R / kBM * kBM;
+    R = R / kRowPad * kRowPad;
     if (R > L.n_pad) R = L.n_pad;
-    if (R < kBM) return MC_ERR_WORKSPACE;
+    if (R < kRowPad) return MC_ERR_WORKSPACE;
   }
   int sms = 0;
   mc_status st = device_info(&sms);
@@ -328,7 +362,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
   if ((e = mc::launch_select_gather(sa, s)) != cudaSuccess) return cuda_fail(e, "row selection launch");
 
   CUtensorMap tm_w_k, tm_w_mn;
-  if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, kBN)) != MC_OK) return st;
+  if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, b_box_rows())) != MC_OK) return st;
   if ((st = make_tmap(&tm_w_mn, w_vocab, d, V, d, 64)) != MC_OK) return st;
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
 
@@ -351,12 +385,13 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.d = d;
     za.V = V;
     za.inv_temperature = inv_temperature;
-    za.splits = choose_splits(ceil_div(rows, kBM), n_tiles, sms);
+    za.splits = choose_splits(ceil_div(rows, row_block()), n_tiles, concurrent_units(sms));
     za.dz = dz;
     za.ld = vp;
     za.ws_status = ws_status;
     za.grid = sms;
     za.timeout_ns = tmo;
+    za.pair = use_pair_engine() ? 1 : 0;
     if ((e = mc::launch_dz(za, s)) != cudaSuccess) return cuda_fail(e, "dZ launch");
 
     mc::DhArgs ha;
@@ -372,6 +407,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     ha.ws_status = ws_status;
     ha.grid = sms;
     ha.timeout_ns = tmo;
+    ha.pair = use_pair_engine() ? 1 : 0;
     if ((e = mc::launch_dh(ha, s)) != cudaSuccess) return cuda_fail(e, "dH launch");
 
     mc::DwArgs wa;
@@ -387,6 +423,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     wa.ws_status = ws_status;
     wa.grid = sms;
     wa.timeout_ns = tmo;
+    wa.pair = use_pair_engine() ? 1 : 0;
     if ((e = mc::launch_dw(wa, s)) != cudaSuccess) return cuda_fail(e, "dW launch");
   }
   if ((e = mc::launch_status_merge(ws_status, dev_status, s)) != cudaSuccess) return cuda_fail(e, "status launch");

@@ -4,7 +4,7 @@
 // (row_keep[t] == 0, i.e. M_i = 0 in Eq. 17, or g_t = gH_t = 0, or an invalid
 // target) contribute nothing; one CTA scans the rows in order and writes the
 // indices of the others (idx[], count). Their hidden rows are gathered into a
-// dense block Hc, zero-padded to a multiple of 128 rows. All later extents come
+// dense block Hc, zero-padded to a multiple of 256 rows. All later extents come
 // from the device-side count, so nothing waits on the host.
 // Stage 1 (dZ producer): the forward's tensor-core mainloop recomputes each
 // 128 x 256 logit tile of the selected rows in TMEM; the epilogue turns it into
@@ -17,6 +17,7 @@
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
+#include "mc_gemm2.cuh"
 #include "mc_internal.h"
 
 namespace mc {
@@ -80,11 +81,12 @@ __global__ void __launch_bounds__(kSelectThreads) select_rows_kernel(
   if (tid == 0) *count = base;
 }
 
-// Hc[j] = H[idx[j]] for j < count, zero rows up to the next multiple of 128.
+// Hc[j] = H[idx[j]] for j < count, zero rows up to the next multiple of 256
+// (a whole row block of either engine).
 __global__ void gather_rows_kernel(const uint4* __restrict__ H, int row_vec, const int32_t* __restrict__ idx,
                                    const int32_t* __restrict__ count, uint4* __restrict__ Hc) {
   const long long cnt = *count;
-  const long long lim = (cnt + BM - 1) / BM * BM;
+  const long long lim = (cnt + PAIR_BM - 1) / PAIR_BM * PAIR_BM;
   for (long long j = blockIdx.x; j < lim; j += gridDim.x) {
     uint4* dst = Hc + j * row_vec;
     if (j < cnt) {
@@ -98,21 +100,26 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ H, int row_vec, con
 
 // ---------------------------------------------------------------- stage 1
 
+struct DzParams {
+  const int32_t* targets;
+  const float* lse;
+  const float* entropy;
+  const float* grad_logp;
+  const float* grad_entropy;
+  const int32_t* idx;  // compacted row -> original row (this chunk's slice)
+  long long rows;      // rows of this chunk (host bound; the device count may be lower)
+  int V;
+  float scale2;
+  float inv_temp;
+  __nv_bfloat16* dz;
+  long long ld;
+};
+
+// kEntropy = false when there is no entropy gradient (gH == 0 for every row):
+// then dZ = -g p everywhere except the target column, which gets g (1 - p).
+template <bool kEntropy>
 struct DzEpi {
-  struct Params {
-    const int32_t* targets;
-    const float* lse;
-    const float* entropy;
-    const float* grad_logp;
-    const float* grad_entropy;
-    const int32_t* idx;  // compacted row -> original row (this chunk's slice)
-    long long rows;      // rows of this chunk (host bound; the device count may be lower)
-    int V;
-    float scale2;
-    float inv_temp;
-    __nv_bfloat16* dz;
-    long long ld;
-  };
+  using Params = DzParams;
 
   long long rows_lim;
   float lse2, cg, cgh, hrow;
@@ -149,17 +156,31 @@ struct DzEpi {
       uint32_t w[16];
       if (valid) {
         const float nl = -lse2;
+        if (kEntropy) {
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          float d2[2];
+          for (int i = 0; i < 32; i += 2) {
+            float d2[2];
 #pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            const float a = fmaf(x[i + j], p.scale2, nl);  // log2 p
-            const float pr = ex2_approx(a);
-            const float oh = (vc + i + j == y) ? 1.f : 0.f;
-            d2[j] = fmaf(cg, oh - pr, -cgh * pr * fmaf(a, kLn2, hrow));
+            for (int j = 0; j < 2; ++j) {
+              const float a = fmaf(x[i + j], p.scale2, nl);  // log2 p
+              const float pr = ex2_approx(a);
+              const float oh = (vc + i + j == y) ? 1.f : 0.f;
+              d2[j] = fmaf(cg, oh - pr, -cgh * pr * fmaf(a, kLn2, hrow));
+            }
+            w[i / 2] = pack_bf16x2(d2[0], d2[1]);
           }
-          w[i / 2] = pack_bf16x2(d2[0], d2[1]);
+        } else {
+          const float ncg = -cg;
+          float dv[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) dv[i] = ncg * ex2_approx(fmaf(x[i], p.scale2, nl));
+          const int rel = y - vc;
+          if (rel >= 0 && rel < 32) {  // the target column of this row lies in this chunk
+#pragma unroll
+            for (int i = 0; i < 32; ++i) dv[i] = (i == rel) ? dv[i] + cg : dv[i];
+          }
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) w[i / 2] = pack_bf16x2(dv[i], dv[i + 1]);
         }
       } else {
 #pragma unroll
@@ -263,7 +284,8 @@ struct StoreF32Epi {
 template <class Epi, bool A_MN, bool B_MN>
 cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedule& sch,
                      const typename Epi::Params& ep, int grid_cap, uint64_t timeout_ns, int32_t* status,
-                     cudaStream_t stream) {
+                     cudaStream_t stream, int pair) {
+  if (pair) return run_gemm_pair<Epi, A_MN, B_MN>(ta, tb, sch, ep, timeout_ns, status, stream);
   auto kern = gemm_persistent<Epi, A_MN, B_MN>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(GEMM_SMEM_BYTES));
@@ -294,7 +316,8 @@ cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   Schedule sch;
-  sch.m_blocks = static_cast<int>((a.rows + BM - 1) / BM);
+  const int rb = a.pair ? PAIR_BM : BM;
+  sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
   sch.k_blocks = a.d / BK;
@@ -302,7 +325,7 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
   sch.dyn_mode = DYN_ROWS;
-  DzEpi::Params ep;
+  DzParams ep;
   ep.targets = a.targets;
   ep.lse = a.lse;
   ep.entropy = a.entropy;
@@ -315,13 +338,17 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   ep.inv_temp = a.inv_temperature;
   ep.dz = static_cast<__nv_bfloat16*>(a.dz);
   ep.ld = a.ld;
-  return run_gemm<DzEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                       stream);
+  if (a.grad_entropy != nullptr)
+    return run_gemm<DzEpi<true>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
+                                               stream, a.pair);
+  return run_gemm<DzEpi<false>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
+                                              stream, a.pair);
 }
 
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   Schedule sch;
-  sch.m_blocks = static_cast<int>((a.rows + BM - 1) / BM);
+  const int rb = a.pair ? PAIR_BM : BM;
+  sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;  // one output tile per unit
   sch.k_blocks = (a.V + BK - 1) / BK;
@@ -336,12 +363,13 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   ep.rows = a.rows;
   ep.cols = a.d;
   return run_gemm<StoreBf16Epi, false, true>(a.tm_dz, a.tm_w_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                             stream);
+                                             stream, a.pair);
 }
 
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   Schedule sch;
-  sch.m_blocks = (a.V + BM - 1) / BM;
+  const int rb = a.pair ? PAIR_BM : BM;
+  sch.m_blocks = (a.V + rb - 1) / rb;
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;
   sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);
@@ -356,7 +384,7 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   ep.cols = a.d;
   ep.accumulate = a.accumulate;
   return run_gemm<StoreF32Epi, true, true>(a.tm_dz_mn, a.tm_h_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                           stream);
+                                           stream, a.pair);
 }
 
 cudaError_t launch_status_merge(const int32_t* ws_status, int32_t* dev_status, cudaStream_t stream) {

@@ -16,6 +16,7 @@
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
+#include "mc_gemm2.cuh"
 #include "mc_internal.h"
 
 namespace mc {
@@ -165,12 +166,10 @@ __global__ void fwd_finalize(const int32_t* __restrict__ targets, long long N, i
 size_t gemm_smem_bytes() { return GEMM_SMEM_BYTES; }
 
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
-  auto kern = gemm_persistent<FwdEpi, false, false>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(GEMM_SMEM_BYTES));
-  if (e != cudaSuccess) return e;
+  cudaError_t e;
   Schedule sch;
-  sch.m_blocks = static_cast<int>((a.N + BM - 1) / BM);
+  const int row_block = a.pair ? PAIR_BM : BM;
+  sch.m_blocks = static_cast<int>((a.N + row_block - 1) / row_block);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
   sch.k_blocks = a.d / BK;
@@ -184,11 +183,18 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   ep.zy = a.zy;
   ep.n_pad = a.n_pad;
   ep.splits = a.splits;
-  const int units = sch.m_blocks * sch.splits;
-  const int grid = units < a.grid ? units : a.grid;
-  kern<<<grid, GEMM_THREADS, GEMM_SMEM_BYTES, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns,
-                                                       a.ws_status);
-  e = cudaGetLastError();
+  if (a.pair) {
+    e = run_gemm_pair<FwdEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
+  } else {
+    auto kern = gemm_persistent<FwdEpi, false, false>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(GEMM_SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    const int units = sch.m_blocks * sch.splits;
+    const int grid = units < a.grid ? units : a.grid;
+    kern<<<grid, GEMM_THREADS, GEMM_SMEM_BYTES, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns,
+                                                         a.ws_status);
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess) return e;
   const int threads = 256;
   const long long blocks = (a.N + threads - 1) / threads;

@@ -29,6 +29,7 @@ struct FwdArgs {
   int32_t* dev_status;
   int grid;
   uint64_t timeout_ns;
+  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream);
 
@@ -70,6 +71,7 @@ struct DzArgs {
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
+  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream);
 
@@ -85,6 +87,7 @@ struct DhArgs {           // grad_hidden[idx[j], :] = (dZ . W)[j, :]
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
+  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream);
 
@@ -100,6 +103,7 @@ struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . Hc[rows, d]
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
+  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream);
 
