@@ -14,6 +14,8 @@ Modules
 ``oracle.filter``    per-sequence signed / absolute mean log importance ratio,
                      the MirrorPop keep-mask (Eq. 18-21, §4.5.2) and per-token
                      ratios (Eq. 4).
+``oracle.grpo``      the masked GRPO clipped-surrogate loss (Eq. 5 / Eq. 17,
+                     without the KL term) and its gradient.
 
 Every function names the passage it follows. Parity is pinned for every
 function by the ``-m "not gpu"`` tests in ``tests/test_oracle_*.py`` (brute
@@ -23,3 +25,4 @@ paper's worked example); none is "parity unpinned".
 
 from .logprobs import logits, token_logprobs, token_logprobs_bwd  # noqa: F401
 from .filter import seq_ratio_filter  # noqa: F401
+from .grpo import grpo_masked_loss  # noqa: F401
