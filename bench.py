@@ -382,13 +382,57 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_stream(args):
+    """HBM bandwidth of the two token-streaming kernels (MirrorPop filter and
+    masked GRPO loss) on a large synthetic batch: 64M tokens in 16,384
+    sequences of 4,096 (or --rows tokens), CUDA events over --launches calls.
+    Algorithmic bytes per token: filter 4 + 4 + 1 read, 4 + 1 written;
+    loss 4 + 4 + 1 read, 4 written (per-sequence arrays are negligible)."""
+    from paper_2606_04847_gb300 import build as mcbuild
+    from paper_2606_04847_gb300 import mc
+
+    torch.cuda.set_device(0)
+    if not os.path.exists(mc.lib_path()):
+        mcbuild.build()
+    N = args.rows if args.rows > 0 else 64 * 1024 * 1024
+    B = 16384
+    g = torch.Generator(device="cuda").manual_seed(0)
+    lp = -torch.rand(N, generator=g, device="cuda") * 8
+    lb = lp + torch.randn(N, generator=g, device="cuda") * 0.2
+    mask = (torch.rand(N, generator=g, device="cuda") < 0.9).to(torch.uint8)
+    cu = torch.linspace(0, N, B + 1, device="cuda").round().to(torch.int64)
+    adv = torch.randn(B, generator=g, device="cuda")
+    flt = mc.seq_ratio_filter(lp, lb, mask, cu, 0.2, 0.2)
+    loss = mc.grpo_masked_loss(lp, lb, mask, cu, adv, flt["keep"], flt["n_tokens"], 0.2, 0.28)
+    peaks = _peaks()
+    res = {"case": "stream", "tokens": N, "sequences": B, "launches": args.launches,
+           "hbm_peak_gbs": peaks["hbm_gbs"], "peak_source": peaks["source"]}
+    for name, fn, bpt in (("filter", lambda: mc.seq_ratio_filter(lp, lb, mask, cu, 0.2, 0.2, out=flt), 14),
+                          ("loss", lambda: mc.grpo_masked_loss(lp, lb, mask, cu, adv, flt["keep"], flt["n_tokens"],
+                                                               0.2, 0.28, out=loss), 13)):
+        fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(args.launches):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / args.launches
+        gbs = bpt * N / (ms / 1e3) / 1e9
+        res[name] = {"ms": ms, "bytes_per_token": bpt, "achieved_gbs": gbs, "frac": gbs / peaks["hbm_gbs"]}
+    print(json.dumps(res), flush=True)
+
+
 def run_case(args):
     """One call of the path, `--launches` times, for ncu captures (no timing printed
-    beyond a one-line summary): --case fwd|bwd|filter on the first `--rows`
+    beyond a one-line summary): --case fwd|bwd|filter|loss on the first `--rows`
     tokens of the workload (0 = all)."""
     from paper_2606_04847_gb300 import build as mcbuild
     from paper_2606_04847_gb300 import mc, workloads
 
+    if args.case == "stream":
+        return run_stream(args)
     torch.cuda.set_device(0)
     if not os.path.exists(mc.lib_path()):
         mcbuild.build()
@@ -408,6 +452,9 @@ def run_case(args):
             mc.token_logprobs(h, w, y, out=fw)
         elif args.case == "filter":
             mc.seq_ratio_filter(fw["logp"], lb, None, cu, spec.delta, spec.delta)
+        elif args.case == "loss":
+            mc.grpo_masked_loss(fw["logp"], lb, None, cu, adv[:1].contiguous(), flt["keep"], flt["n_tokens"],
+                                0.2, 0.28)
         else:  # every row live, so the capture does not depend on whether the filter keeps this slice
             mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], adv, None)
     torch.cuda.synchronize()
@@ -465,7 +512,7 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=384)
     ap.add_argument("--ref-rows", type=int, default=64)
-    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter"], default="step",
+    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream"], default="step",
                     help="profiling aid: run one call of the path --launches times")
     ap.add_argument("--rows", type=int, default=0, help="--case: tokens to use (0 = the whole batch)")
     ap.add_argument("--launches", type=int, default=2)

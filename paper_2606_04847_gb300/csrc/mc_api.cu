@@ -468,6 +468,57 @@ mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behavi
   return MC_OK;
 }
 
+size_t mc_grpo_masked_loss_workspace_size(int32_t B) {
+  if (B < 1) return 0;
+  return kStatusBytes + align_up(size_t(B) * sizeof(float), 256);
+}
+
+mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behaviour, const uint8_t* loss_mask,
+                              const int64_t* cu_seqlens, const float* advantages, const uint8_t* keep,
+                              const int32_t* n_tokens, int32_t B, int64_t N, float eps_low, float eps_high,
+                              float* loss, float* grad_logp, float* seq_loss, int32_t* n_clipped, void* workspace,
+                              size_t workspace_bytes, mc_stream_t stream) {
+  if (B < 1 || N < 0 || N >= (1LL << 40)) return MC_ERR_INVALID_ARG;
+  if (!(eps_low >= 0.f && eps_low < 1.f) || !(eps_high >= 0.f) || !std::isfinite(eps_high))
+    return MC_ERR_INVALID_ARG;
+  if (!cu_seqlens || !advantages || !keep || !n_tokens || !loss) return MC_ERR_INVALID_ARG;
+  if (N > 0 && (!logp_policy || !logp_behaviour || !grad_logp)) return MC_ERR_INVALID_ARG;
+  if (!aligned(cu_seqlens, 8) || !aligned(advantages, 4) || !aligned(n_tokens, 4) || !aligned(loss, 4) ||
+      (logp_policy && !aligned(logp_policy, 4)) || (logp_behaviour && !aligned(logp_behaviour, 4)) ||
+      (grad_logp && !aligned(grad_logp, 4)) || (seq_loss && !aligned(seq_loss, 4)) ||
+      (n_clipped && !aligned(n_clipped, 4)))
+    return MC_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < mc_grpo_masked_loss_workspace_size(B))
+    return MC_ERR_WORKSPACE;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  mc::LossArgs a;
+  a.logp_policy = logp_policy;
+  a.logp_behaviour = logp_behaviour;
+  a.loss_mask = loss_mask;
+  a.cu_seqlens = cu_seqlens;
+  a.advantages = advantages;
+  a.keep = keep;
+  a.n_tokens = n_tokens;
+  a.B = B;
+  a.N = N;
+  a.eps_low = eps_low;
+  a.eps_high = eps_high;
+  a.loss = loss;
+  a.grad_logp = grad_logp;
+  a.seq_loss = seq_loss;
+  a.n_clipped = n_clipped;
+  a.Z = reinterpret_cast<long long*>(ws);
+  a.seq_share = reinterpret_cast<float*>(ws + kStatusBytes);
+  a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && aligned(grad_logp, 16) &&
+             (!loss_mask || aligned(loss_mask, 4));
+  cudaError_t e = mc::launch_grpo_loss(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "GRPO loss launch");
+  return MC_OK;
+}
+
 mc_status mc_selftest_bounded_wait(int32_t* dev_status, int64_t timeout_ns, mc_stream_t stream) {
   if (!dev_status || !aligned(dev_status, 4)) return MC_ERR_INVALID_ARG;
   if (timeout_ns < 1000000LL || timeout_ns > 10000000000LL) return MC_ERR_INVALID_ARG;

@@ -129,6 +129,27 @@ struct FilterArgs {
 };
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream);
 
+struct LossArgs {
+  const float* logp_policy;
+  const float* logp_behaviour;
+  const uint8_t* loss_mask;
+  const int64_t* cu_seqlens;
+  const float* advantages;
+  const uint8_t* keep;
+  const int32_t* n_tokens;
+  int B;
+  long long N;
+  float eps_low, eps_high;
+  float* loss;
+  float* grad_logp;
+  float* seq_loss;
+  int32_t* n_clipped;
+  long long* Z;           // workspace
+  float* seq_share;       // workspace [B]
+  int vec_ok;
+};
+cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream);
+
 cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream);
 
 size_t gemm_smem_bytes();

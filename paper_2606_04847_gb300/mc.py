@@ -49,6 +49,8 @@ SIGNATURES = {
     "mc_token_logprobs_bwd": (_I32, [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _I32, _P,
                                      _SZ, _P, _P]),
     "mc_seq_ratio_filter": (_I32, [_P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _P, _P, _P]),
+    "mc_grpo_masked_loss_workspace_size": (_SZ, [_I32]),
+    "mc_grpo_masked_loss": (_I32, [_P, _P, _P, _P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _SZ, _P]),
     "mc_selftest_bounded_wait": (_I32, [_P, _I64, _P]),
 }
 
@@ -231,6 +233,38 @@ def seq_ratio_filter(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
                                    _ptr(out.get("keep_vanilla")), _ptr(out.get("token_ratio")),
                                    _ptr(out.get("token_keep")), _stream(stream))
     _check("mc_seq_ratio_filter", st)
+    return out
+
+
+def grpo_masked_loss(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, loss_mask: Optional[torch.Tensor],
+                     cu_seqlens: torch.Tensor, advantages: torch.Tensor, keep: torch.Tensor, n_tokens: torch.Tensor,
+                     eps_low: float, eps_high: float, *, out: Optional[dict] = None,
+                     workspace: Optional[torch.Tensor] = None, stream=None) -> dict:
+    """mc_grpo_masked_loss: {"loss" [1], "grad_logp" [N], "seq_loss" [B], "n_clipped" [1]}."""
+    _need(logp_policy, "logp_policy", torch.float32, 1)
+    _need(logp_behaviour, "logp_behaviour", torch.float32, 1)
+    _need(cu_seqlens, "cu_seqlens", torch.int64, 1)
+    _need(advantages, "advantages", torch.float32, 1)
+    _need(keep, "keep", torch.uint8, 1)
+    _need(n_tokens, "n_tokens", torch.int32, 1)
+    if loss_mask is not None:
+        _need(loss_mask, "loss_mask", torch.uint8, 1)
+    N = logp_policy.shape[0]
+    B = cu_seqlens.shape[0] - 1
+    dev = logp_policy.device
+    if out is None:
+        out = {"loss": torch.empty(1, dtype=torch.float32, device=dev),
+               "grad_logp": torch.empty(N, dtype=torch.float32, device=dev),
+               "seq_loss": torch.empty(B, dtype=torch.float32, device=dev),
+               "n_clipped": torch.empty(1, dtype=torch.int32, device=dev)}
+    if workspace is None:
+        workspace = torch.empty(lib().mc_grpo_masked_loss_workspace_size(B), dtype=torch.uint8, device=dev)
+    st = lib().mc_grpo_masked_loss(_ptr(logp_policy), _ptr(logp_behaviour), _ptr(loss_mask), _ptr(cu_seqlens),
+                                   _ptr(advantages), _ptr(keep), _ptr(n_tokens), B, N, float(eps_low),
+                                   float(eps_high), _ptr(out["loss"]), _ptr(out["grad_logp"]),
+                                   _ptr(out.get("seq_loss")), _ptr(out.get("n_clipped")), _ptr(workspace),
+                                   workspace.numel(), _stream(stream))
+    _check("mc_grpo_masked_loss", st)
     return out
 
 

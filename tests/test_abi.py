@@ -125,6 +125,23 @@ def test_filter_argument_checks(L):
     assert filt(L, cu=FAKE + 4) == INVALID  # int64 array not 8-byte aligned
 
 
+def loss_call(L, B=2, N=10, eps_low=0.2, eps_high=0.2, keep=FAKE, ws=FAKE, ws_bytes=1 << 20):
+    return L.mc_grpo_masked_loss(FAKE, FAKE, None, FAKE, FAKE, keep, FAKE, B, N, eps_low, eps_high, FAKE, FAKE,
+                                 None, None, ws, ws_bytes, None)
+
+
+def test_loss_argument_checks(L):
+    assert L.mc_grpo_masked_loss_workspace_size(0) == 0
+    assert L.mc_grpo_masked_loss_workspace_size(1000) >= 256 + 4000
+    assert loss_call(L, B=0) == INVALID
+    assert loss_call(L, eps_low=1.0) == INVALID
+    assert loss_call(L, eps_low=-0.1) == INVALID
+    assert loss_call(L, eps_high=float("inf")) == INVALID
+    assert loss_call(L, keep=None) == INVALID
+    assert loss_call(L, ws=None) == WORKSPACE
+    assert loss_call(L, ws_bytes=16) == WORKSPACE
+
+
 def test_selftest_argument_checks(L):
     assert L.mc_selftest_bounded_wait(None, 10 ** 8, None) == INVALID
     assert L.mc_selftest_bounded_wait(FAKE, 10, None) == INVALID
