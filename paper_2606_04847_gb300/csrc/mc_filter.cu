@@ -1,10 +1,12 @@
 // mc_filter.cu — per-sequence importance-ratio statistics and the MirrorPop
 // keep-mask (§4.5.2, Eq. 18-21), plus per-token ratios (Eq. 4).
 //
-// One CTA per sequence. Each thread walks its share of the sequence's packed
-// tokens with 16-byte loads (4 tokens of logp_policy / logp_behaviour, 4 mask
-// bytes), accumulates sum(log rho), sum(|log rho|) and the count over loss-
-// masked tokens, and writes rho = exp(log rho) on the way. Warp shuffles then
+// Persistent CTAs (8 per SM) stride over the sequences, one sequence at a
+// time per CTA. Each thread walks its share of the sequence's packed tokens
+// with 16-byte loads (4 tokens of logp_policy / logp_behaviour, 4 mask bytes;
+// two vectors in flight), accumulates sum(log rho), sum(|log rho|) and the
+// count over loss-masked tokens, and writes rho = exp(log rho) on the way
+// (streaming stores). Warp shuffles then
 // a shared-memory step reduce the three sums in a fixed order (deterministic
 // for a given launch shape). Thread 0 forms the statistics and the masks; a
 // second sweep writes token_keep once keep_i is known. The kernel is HBM-
@@ -33,78 +35,99 @@ __device__ __forceinline__ void add_token(Acc& acc, float lp, float lb, bool m, 
   }
 }
 
+__device__ __forceinline__ void add_vec(Acc& acc, const float4& lp, const float4& lb, uchar4 mk, float* ratio_out) {
+  const float d0 = lp.x - lb.x, d1 = lp.y - lb.y, d2 = lp.z - lb.z, d3 = lp.w - lb.w;
+  if (ratio_out) __stcs(reinterpret_cast<float4*>(ratio_out), make_float4(__expf(d0), __expf(d1), __expf(d2), __expf(d3)));
+  if (mk.x) { acc.s += d0; acc.a += fabsf(d0); acc.n += 1; }
+  if (mk.y) { acc.s += d1; acc.a += fabsf(d1); acc.n += 1; }
+  if (mk.z) { acc.s += d2; acc.a += fabsf(d2); acc.n += 1; }
+  if (mk.w) { acc.s += d3; acc.a += fabsf(d3); acc.n += 1; }
+}
+
+// Persistent over sequences (CTA c handles sequences c, c + gridDim.x, ...).
 __global__ void __launch_bounds__(kFilterThreads) seq_filter_kernel(FilterArgs p) {
-  const int i = blockIdx.x;
-  long long b = p.cu_seqlens[i];
-  long long e = p.cu_seqlens[i + 1];
-  // Clamp the segment to [0, N) so malformed cu_seqlens cannot index out of bounds.
-  b = b < 0 ? 0 : (b > p.N ? p.N : b);
-  e = e < b ? b : (e > p.N ? p.N : e);
-
-  Acc acc{0.f, 0.f, 0};
-  // Scalar head up to a multiple of 4 tokens, then 4-token vectors, then the tail.
-  // (p.vec_ok = 0 when some pointer is not aligned for vector access: all scalar.)
-  long long hb = p.vec_ok ? ((b + 3) & ~3LL) : e;
-  if (hb > e) hb = e;
-  const long long vend = hb + ((e - hb) & ~3LL);
-  for (long long t = b + threadIdx.x; t < hb; t += blockDim.x)
-    add_token(acc, p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true,
-              p.token_ratio ? p.token_ratio + t : nullptr);
-  for (long long t = hb + 4LL * threadIdx.x; t < vend; t += 4LL * blockDim.x) {
-    const float4 lp = *reinterpret_cast<const float4*>(p.logp_policy + t);
-    const float4 lb = *reinterpret_cast<const float4*>(p.logp_behaviour + t);
-    uchar4 mk = make_uchar4(1, 1, 1, 1);
-    if (p.loss_mask) mk = *reinterpret_cast<const uchar4*>(p.loss_mask + t);
-    const float d0 = lp.x - lb.x, d1 = lp.y - lb.y, d2 = lp.z - lb.z, d3 = lp.w - lb.w;
-    if (p.token_ratio)
-      *reinterpret_cast<float4*>(p.token_ratio + t) = make_float4(__expf(d0), __expf(d1), __expf(d2), __expf(d3));
-    if (mk.x) { acc.s += d0; acc.a += fabsf(d0); acc.n += 1; }
-    if (mk.y) { acc.s += d1; acc.a += fabsf(d1); acc.n += 1; }
-    if (mk.z) { acc.s += d2; acc.a += fabsf(d2); acc.n += 1; }
-    if (mk.w) { acc.s += d3; acc.a += fabsf(d3); acc.n += 1; }
-  }
-  for (long long t = vend + threadIdx.x; t < e; t += blockDim.x)
-    add_token(acc, p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true,
-              p.token_ratio ? p.token_ratio + t : nullptr);
-
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    acc.s += __shfl_xor_sync(0xffffffffu, acc.s, off);
-    acc.a += __shfl_xor_sync(0xffffffffu, acc.a, off);
-    acc.n += __shfl_xor_sync(0xffffffffu, acc.n, off);
-  }
   __shared__ Acc warp_acc[kFilterThreads / 32];
   __shared__ int keep_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) warp_acc[warp] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    Acc tot{0.f, 0.f, 0};
-    for (int w = 0; w < kFilterThreads / 32; ++w) {
-      tot.s += warp_acc[w].s;
-      tot.a += warp_acc[w].a;
-      tot.n += warp_acc[w].n;
+  for (int i = blockIdx.x; i < p.B; i += gridDim.x) {
+    long long b = p.cu_seqlens[i];
+    long long e = p.cu_seqlens[i + 1];
+    // Clamp the segment to [0, N) so malformed cu_seqlens cannot index out of bounds.
+    b = b < 0 ? 0 : (b > p.N ? p.N : b);
+    e = e < b ? b : (e > p.N ? p.N : e);
+
+    Acc acc{0.f, 0.f, 0};
+    // Scalar head up to a multiple of 4 tokens, then 4-token vectors (two in
+    // flight per thread: both loads issue before either is used), then the tail.
+    // (p.vec_ok = 0 when some pointer is not aligned for vector access: all scalar.)
+    long long hb = p.vec_ok ? ((b + 3) & ~3LL) : e;
+    if (hb > e) hb = e;
+    const long long vend = hb + ((e - hb) & ~3LL);
+    for (long long t = b + threadIdx.x; t < hb; t += blockDim.x)
+      add_token(acc, p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true,
+                p.token_ratio ? p.token_ratio + t : nullptr);
+    const long long q1 = vend >> 2;
+    const float4* lp4 = reinterpret_cast<const float4*>(p.logp_policy);
+    const float4* lb4 = reinterpret_cast<const float4*>(p.logp_behaviour);
+    const uchar4* m4 = reinterpret_cast<const uchar4*>(p.loss_mask);
+    for (long long q = (hb >> 2) + threadIdx.x; q < q1; q += 2LL * blockDim.x) {
+      const long long r = q + blockDim.x;
+      const bool two = r < q1;
+      const float4 lp0 = __ldcs(lp4 + q);
+      const float4 lb0 = __ldcs(lb4 + q);
+      const uchar4 m0 = p.loss_mask ? m4[q] : make_uchar4(1, 1, 1, 1);
+      float4 lp1 = make_float4(0.f, 0.f, 0.f, 0.f), lb1 = lp1;
+      uchar4 m1 = make_uchar4(0, 0, 0, 0);
+      if (two) {
+        lp1 = __ldcs(lp4 + r);
+        lb1 = __ldcs(lb4 + r);
+        m1 = p.loss_mask ? m4[r] : make_uchar4(1, 1, 1, 1);
+      }
+      add_vec(acc, lp0, lb0, m0, p.token_ratio ? p.token_ratio + 4 * q : nullptr);
+      if (two) add_vec(acc, lp1, lb1, m1, p.token_ratio ? p.token_ratio + 4 * r : nullptr);
     }
-    float S = 0.f, A = 0.f;
-    int keep = 0, keep_v = 0;
-    if (tot.n > 0) {
-      S = tot.s / static_cast<float>(tot.n);
-      A = tot.a / static_cast<float>(tot.n);
-      keep = A <= p.delta ? 1 : 0;                                   // Eq. 21
-      keep_v = (p.delta_vanilla >= 0.f && fabsf(S) <= p.delta_vanilla) ? 1 : 0;
+    for (long long t = vend + threadIdx.x; t < e; t += blockDim.x)
+      add_token(acc, p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true,
+                p.token_ratio ? p.token_ratio + t : nullptr);
+
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      acc.s += __shfl_xor_sync(0xffffffffu, acc.s, off);
+      acc.a += __shfl_xor_sync(0xffffffffu, acc.a, off);
+      acc.n += __shfl_xor_sync(0xffffffffu, acc.n, off);
     }
-    p.signed_mean[i] = S;
-    p.abs_mean[i] = A;
-    p.n_tokens[i] = tot.n;
-    p.keep[i] = static_cast<uint8_t>(keep);
-    if (p.keep_vanilla) p.keep_vanilla[i] = static_cast<uint8_t>(keep_v);
-    keep_s = keep;
+    if (lane == 0) warp_acc[warp] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      Acc tot{0.f, 0.f, 0};
+      for (int w = 0; w < kFilterThreads / 32; ++w) {
+        tot.s += warp_acc[w].s;
+        tot.a += warp_acc[w].a;
+        tot.n += warp_acc[w].n;
+      }
+      float S = 0.f, A = 0.f;
+      int keep = 0, keep_v = 0;
+      if (tot.n > 0) {
+        S = tot.s / static_cast<float>(tot.n);
+        A = tot.a / static_cast<float>(tot.n);
+        keep = A <= p.delta ? 1 : 0;                                   // Eq. 21
+        keep_v = (p.delta_vanilla >= 0.f && fabsf(S) <= p.delta_vanilla) ? 1 : 0;
+      }
+      p.signed_mean[i] = S;
+      p.abs_mean[i] = A;
+      p.n_tokens[i] = tot.n;
+      p.keep[i] = static_cast<uint8_t>(keep);
+      if (p.keep_vanilla) p.keep_vanilla[i] = static_cast<uint8_t>(keep_v);
+      keep_s = keep;
+    }
+    __syncthreads();
+    if (p.token_keep != nullptr) {
+      const uint8_t k = static_cast<uint8_t>(keep_s);
+      for (long long t = b + threadIdx.x; t < e; t += blockDim.x)
+        p.token_keep[t] = static_cast<uint8_t>(k & (p.loss_mask ? (p.loss_mask[t] != 0) : 1));
+    }
+    __syncthreads();  // warp_acc / keep_s are reused by the next sequence
   }
-  if (p.token_keep == nullptr) return;
-  __syncthreads();
-  const uint8_t k = static_cast<uint8_t>(keep_s);
-  for (long long t = b + threadIdx.x; t < e; t += blockDim.x)
-    p.token_keep[t] = static_cast<uint8_t>(k & (p.loss_mask ? (p.loss_mask[t] != 0) : 1));
 }
 
 // Waits on a barrier nothing arrives at, through the same bounded wait the
@@ -125,7 +148,8 @@ __global__ void selftest_wait_kernel(int32_t* dev_status, uint64_t timeout_ns) {
 
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream) {
   if (a.B <= 0) return cudaSuccess;
-  seq_filter_kernel<<<a.B, kFilterThreads, 0, stream>>>(a);
+  const int grid = a.B < a.grid ? a.B : a.grid;
+  seq_filter_kernel<<<grid, kFilterThreads, 0, stream>>>(a);
   return cudaGetLastError();
 }
 

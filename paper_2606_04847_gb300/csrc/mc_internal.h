@@ -126,6 +126,7 @@ struct FilterArgs {
   float* token_ratio;
   uint8_t* token_keep;
   int vec_ok;             // all float arrays 16-byte and loss_mask 4-byte aligned
+  int grid;               // persistent CTAs (sequences are strided over them)
 };
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream);
 
@@ -147,6 +148,7 @@ struct LossArgs {
   long long* Z;           // workspace
   float* seq_share;       // workspace [B]
   int vec_ok;
+  int grid;               // persistent CTAs (sequences are strided over them)
 };
 cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream);
 

@@ -8,8 +8,9 @@
 //   dL/dlogp_t = -M_i rho_t A_i / Z if rho_t A_i <= the clipped term, else 0
 //
 // Three launches: (1) one CTA forms Z from the filter's keep / n_tokens;
-// (2) one CTA per sequence writes g_t for its tokens (16-byte loads, as the
-// filter) and its share of L; (3) one CTA sums the shares in a fixed order.
+// (2) persistent CTAs stride over the sequences, write g_t for every token
+// (16-byte loads and stores, two vectors in flight per thread) and each
+// response's share of L; (3) one CTA sums the shares in a fixed order.
 // All reductions are fixed-order, so results are bitwise reproducible.
 #include "mc_internal.h"
 #include "mc_ptx.cuh"
@@ -57,59 +58,79 @@ __device__ __forceinline__ float token_grad(float lp, float lb, bool counted, fl
   return clipped ? 0.f : -kz * u;                    // -M_i rho A / Z
 }
 
-__global__ void __launch_bounds__(kLossThreads) grpo_loss_kernel(LossArgs p) {
-  const int i = blockIdx.x;
-  long long b = p.cu_seqlens[i];
-  long long e = p.cu_seqlens[i + 1];
-  b = b < 0 ? 0 : (b > p.N ? p.N : b);
-  e = e < b ? b : (e > p.N ? p.N : e);
-  const long long Z = *p.Z;
-  const float M = (p.keep[i] != 0 && Z > 0) ? 1.f : 0.f;
-  const float A = p.advantages[i];
-  const float kz = Z > 0 ? M / static_cast<float>(Z) : 0.f;
-  const float lo = 1.f - p.eps_low, hi = 1.f + p.eps_high;
+__device__ __forceinline__ float4 vec_grad(const float4& lp, const float4& lb, uchar4 mk, float A, float lo, float hi,
+                                           float kz, TokAcc& acc) {
+  float4 g;
+  g.x = token_grad(lp.x, lb.x, mk.x != 0, A, lo, hi, kz, acc);
+  g.y = token_grad(lp.y, lb.y, mk.y != 0, A, lo, hi, kz, acc);
+  g.z = token_grad(lp.z, lb.z, mk.z != 0, A, lo, hi, kz, acc);
+  g.w = token_grad(lp.w, lb.w, mk.w != 0, A, lo, hi, kz, acc);
+  return g;
+}
 
-  TokAcc acc{0.f, 0};
-  long long hb = p.vec_ok ? ((b + 3) & ~3LL) : e;
-  if (hb > e) hb = e;
-  const long long vend = hb + ((e - hb) & ~3LL);
-  for (long long t = b + threadIdx.x; t < hb; t += blockDim.x)
-    p.grad_logp[t] = token_grad(p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true, A,
-                                lo, hi, kz, acc);
-  for (long long t = hb + 4LL * threadIdx.x; t < vend; t += 4LL * blockDim.x) {
-    const float4 lp = *reinterpret_cast<const float4*>(p.logp_policy + t);
-    const float4 lb = *reinterpret_cast<const float4*>(p.logp_behaviour + t);
-    uchar4 mk = make_uchar4(1, 1, 1, 1);
-    if (p.loss_mask) mk = *reinterpret_cast<const uchar4*>(p.loss_mask + t);
-    float4 g;
-    g.x = token_grad(lp.x, lb.x, mk.x != 0, A, lo, hi, kz, acc);
-    g.y = token_grad(lp.y, lb.y, mk.y != 0, A, lo, hi, kz, acc);
-    g.z = token_grad(lp.z, lb.z, mk.z != 0, A, lo, hi, kz, acc);
-    g.w = token_grad(lp.w, lb.w, mk.w != 0, A, lo, hi, kz, acc);
-    *reinterpret_cast<float4*>(p.grad_logp + t) = g;
-  }
-  for (long long t = vend + threadIdx.x; t < e; t += blockDim.x)
-    p.grad_logp[t] = token_grad(p.logp_policy[t], p.logp_behaviour[t], p.loss_mask ? p.loss_mask[t] != 0 : true, A,
-                                lo, hi, kz, acc);
+__global__ void __launch_bounds__(kLossThreads) grpo_loss_kernel(LossArgs p) {
+  __shared__ TokAcc warp_acc[kLossThreads / 32];
+  const long long Z = *p.Z;
+  const float lo = 1.f - p.eps_low, hi = 1.f + p.eps_high;
+  const float4* lp4 = reinterpret_cast<const float4*>(p.logp_policy);
+  const float4* lb4 = reinterpret_cast<const float4*>(p.logp_behaviour);
+  const uchar4* m4 = reinterpret_cast<const uchar4*>(p.loss_mask);
+  float4* g4 = reinterpret_cast<float4*>(p.grad_logp);
+  for (int i = blockIdx.x; i < p.B; i += gridDim.x) {
+    long long b = p.cu_seqlens[i];
+    long long e = p.cu_seqlens[i + 1];
+    b = b < 0 ? 0 : (b > p.N ? p.N : b);
+    e = e < b ? b : (e > p.N ? p.N : e);
+    const float M = (p.keep[i] != 0 && Z > 0) ? 1.f : 0.f;
+    const float A = p.advantages[i];
+    const float kz = Z > 0 ? M / static_cast<float>(Z) : 0.f;
+
+    TokAcc acc{0.f, 0};
+    long long hb = p.vec_ok ? ((b + 3) & ~3LL) : e;
+    if (hb > e) hb = e;
+    const long long vend = hb + ((e - hb) & ~3LL);
+    for (long long t = b + threadIdx.x; t < hb; t += blockDim.x)
+      p.grad_logp[t] = token_grad(p.logp_policy[t], p.logp_behaviour[t],
+                                  p.loss_mask ? p.loss_mask[t] != 0 : true, A, lo, hi, kz, acc);
+    const long long q1 = vend >> 2;
+    for (long long q = (hb >> 2) + threadIdx.x; q < q1; q += 2LL * blockDim.x) {
+      const long long r = q + blockDim.x;
+      const bool two = r < q1;
+      const float4 lpa = __ldcs(lp4 + q), lba = __ldcs(lb4 + q);
+      const uchar4 ma = p.loss_mask ? m4[q] : make_uchar4(1, 1, 1, 1);
+      float4 lpb = make_float4(0.f, 0.f, 0.f, 0.f), lbb = lpb;
+      uchar4 mb = make_uchar4(0, 0, 0, 0);
+      if (two) {
+        lpb = __ldcs(lp4 + r);
+        lbb = __ldcs(lb4 + r);
+        mb = p.loss_mask ? m4[r] : make_uchar4(1, 1, 1, 1);
+      }
+      __stcs(g4 + q, vec_grad(lpa, lba, ma, A, lo, hi, kz, acc));
+      if (two) __stcs(g4 + r, vec_grad(lpb, lbb, mb, A, lo, hi, kz, acc));
+    }
+    for (long long t = vend + threadIdx.x; t < e; t += blockDim.x)
+      p.grad_logp[t] = token_grad(p.logp_policy[t], p.logp_behaviour[t],
+                                  p.loss_mask ? p.loss_mask[t] != 0 : true, A, lo, hi, kz, acc);
 
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    acc.s += __shfl_xor_sync(0xffffffffu, acc.s, o);
-    acc.clipped += __shfl_xor_sync(0xffffffffu, acc.clipped, o);
-  }
-  __shared__ TokAcc warp_acc[kLossThreads / 32];
-  if ((threadIdx.x & 31) == 0) warp_acc[threadIdx.x >> 5] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    TokAcc tot{0.f, 0};
-    for (int w = 0; w < kLossThreads / 32; ++w) {
-      tot.s += warp_acc[w].s;
-      tot.clipped += warp_acc[w].clipped;
+    for (int o = 16; o > 0; o >>= 1) {
+      acc.s += __shfl_xor_sync(0xffffffffu, acc.s, o);
+      acc.clipped += __shfl_xor_sync(0xffffffffu, acc.clipped, o);
     }
-    const float share = -tot.s * kz;  // this response's share of L
-    p.seq_share[i] = share;
-    if (p.seq_loss) p.seq_loss[i] = share;
-    if (p.n_clipped && M != 0.f && tot.clipped) atomicAdd(p.n_clipped, tot.clipped);
+    if ((threadIdx.x & 31) == 0) warp_acc[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      TokAcc tot{0.f, 0};
+      for (int w = 0; w < kLossThreads / 32; ++w) {
+        tot.s += warp_acc[w].s;
+        tot.clipped += warp_acc[w].clipped;
+      }
+      const float share = -tot.s * kz;  // this response's share of L
+      p.seq_share[i] = share;
+      if (p.seq_loss) p.seq_loss[i] = share;
+      if (p.n_clipped && M != 0.f && tot.clipped) atomicAdd(p.n_clipped, tot.clipped);
+    }
+    __syncthreads();  // warp_acc is reused by the next sequence
   }
 }
 
@@ -135,7 +156,8 @@ cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream) {
   grpo_norm_kernel<<<1, kReduceThreads, 0, stream>>>(a.keep, a.n_tokens, a.B, a.Z, a.n_clipped);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  grpo_loss_kernel<<<a.B, kLossThreads, 0, stream>>>(a);
+  const int grid = a.B < a.grid ? a.B : a.grid;
+  grpo_loss_kernel<<<grid, kLossThreads, 0, stream>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   grpo_final_kernel<<<1, kReduceThreads, 0, stream>>>(a.seq_share, a.B, a.loss);
   return cudaGetLastError();
