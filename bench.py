@@ -42,7 +42,8 @@ if ROOT not in sys.path:
 import torch  # noqa: E402
 
 METRIC = "rollout tokens/sec for fused logprob fwd+bwd at 1 GB300; % of bf16 tensor peak"
-CONFIG_ID = 5
+METRIC_FWD = "rollout tokens/sec for fused logprob fwd + MirrorPop filter at 1 GB300; % of bf16 tensor peak"
+CONFIG_ID = 5  # the fused forward+backward workload the metric names (the default of --config)
 FWD_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fwd_kernel_traffic.json")
 
 
@@ -171,13 +172,14 @@ def oracle_sample_step(wl, rows, delta):
     h = wl.hidden[:rows].cpu()
     w = wl.w_vocab.cpu() if wl.w_vocab.is_cuda else wl.w_vocab
     y = wl.targets[:rows].cpu()
-    adv = wl.advantages[:rows].cpu().double().numpy()
+    adv = None if wl.advantages is None else wl.advantages[:rows].cpu().double().numpy()
     gap = wl.gap[:rows].cpu().double().numpy()
     t0 = time.perf_counter()
     fw = oracle.token_logprobs(h, w, y, 1.0)
     flt = oracle.seq_ratio_filter(fw["logp"], fw["logp"] + gap, None, np.array([0, rows]), delta, delta)
-    g = adv * flt["token_keep"]
-    oracle.token_logprobs_bwd(h, w, y, g, None, 1.0)
+    if adv is not None:  # the forward-only configurations have no backward
+        g = adv * flt["token_keep"]
+        oracle.token_logprobs_bwd(h, w, y, g, None, 1.0)
     return time.perf_counter() - t0
 
 
@@ -198,15 +200,16 @@ def run_ours(args):
     world, rank, local = _dist_setup(args)
     if not os.path.exists(mc.lib_path()):
         mcbuild.build()
-    spec = workloads.spec_for(CONFIG_ID)
+    spec = workloads.spec_for(args.config)
     if world > 1:
-        spec = workloads.spec_for(CONFIG_ID, seed=spec.seed + 1000 * rank)  # each replica its own batch
+        spec = workloads.spec_for(args.config, seed=spec.seed + 1000 * rank)  # each replica its own batch
     wl = workloads.build(spec, "cuda")
     dev = torch.device("cuda")
     N, d, V, B = wl.N, spec.d, spec.V, wl.B
     delta = spec.delta
     h, w, y = wl.hidden, wl.w_vocab, wl.targets
     cu, mask, adv = wl.cu_seqlens, wl.loss_mask, wl.advantages
+    has_bwd = adv is not None  # the forward-only configurations time forward + filter
 
     # Behaviour log-probs: policy log-probs + the per-sequence gap (untimed).
     pre = mc.token_logprobs(h, w, y)
@@ -215,9 +218,10 @@ def run_ours(args):
 
     fw_out = {k: torch.empty(N, dtype=torch.float32, device=dev) for k in ("logp", "entropy", "lse")}
     fw_ws = torch.empty(mc.forward_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
-    bw_ws = torch.empty(mc.backward_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
-    gh = torch.empty((N, d), dtype=torch.bfloat16, device=dev)
-    gw = torch.empty((V, d), dtype=torch.float32, device=dev)
+    if has_bwd:
+        bw_ws = torch.empty(mc.backward_workspace_size(N, d, V), dtype=torch.uint8, device=dev)
+        gh = torch.empty((N, d), dtype=torch.bfloat16, device=dev)
+        gw = torch.empty((V, d), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     ev = {k: [] for k in ("fwd", "filter", "bwd")}
 
@@ -232,8 +236,10 @@ def run_ours(args):
         flt = mc.seq_ratio_filter(fw_out["logp"], lb, mm, cc, delta, delta, stream=stream)
         if record:
             e[2].record(stream)
-        mc.token_logprobs_bwd(hh, w, yy, fw_out["lse"], fw_out["entropy"], aa, None, row_keep=flt["token_keep"],
-                              grad_hidden=gh, grad_w=gw, workspace=bw_ws, stream=stream)
+        if has_bwd:
+            mc.token_logprobs_bwd(hh, w, yy, fw_out["lse"], fw_out["entropy"], aa, None,
+                                  row_keep=flt["token_keep"], grad_hidden=gh, grad_w=gw, workspace=bw_ws,
+                                  stream=stream)
         if record:
             e[3].record(stream)
             ev["fwd"].append((e[0], e[1]))
@@ -267,16 +273,21 @@ def run_ours(args):
     def avg(k):
         return sum(a.elapsed_time(b) for a, b in ev[k]) / len(ev[k])
 
-    t_fwd, t_flt, t_bwd = avg("fwd"), avg("filter"), avg("bwd")
+    t_fwd, t_flt, t_bwd = avg("fwd"), avg("filter"), avg("bwd") if has_bwd else 0.0
     flop_fwd = 2.0 * N * d * V
-    flop_bwd = 4.0 * kept_rows * d * V  # algorithmic: rows with a nonzero upstream gradient
+    flop_bwd = 4.0 * kept_rows * d * V if has_bwd else 0.0  # algorithmic: rows with a nonzero upstream gradient
     peaks = _peaks()
-    peak_tf = peaks["bf16_sustained"]
+    # The sustained (power-capped) figure for a kernel whose clocks the power
+    # cap held down during the timed region, the burst figure otherwise.
+    capped = clk.get("sm_mhz") is None or clk.get("sm_max_mhz") is None or \
+        clk["sm_mhz"] < 0.97 * clk["sm_max_mhz"]
+    peak_tf = peaks["bf16_sustained"] if capped else peaks["bf16"]
+    peak_kind = "sustained" if capped else "burst"
     achieved = flop_fwd / (t_fwd / 1e3) / 1e12
     traffic = None
     if os.path.exists(FWD_TRAFFIC_FILE):
         tj = json.load(open(FWD_TRAFFIC_FILE))
-        if tj.get("kernel_source_hash") == _kernel_source_hash():
+        if tj.get("kernel_source_hash") == _kernel_source_hash() and tj.get("config", 5) == args.config:
             traffic = tj["bytes_per_full_launch"] * (N / tj["full_launch_rows"])
     step_tflops = (flop_fwd + flop_bwd) * args.steps / (ms / 1e3) / 1e12
 
@@ -288,7 +299,7 @@ def run_ours(args):
         # overlaps the kernels of step i; the per-token and per-sequence
         # results of every step are read back to pinned host memory. All of
         # it, including the first copy, lies inside the timed region.
-        host = [t.cpu().pin_memory() for t in (h, y, logp_b, mask, cu, adv)]
+        host = [t.cpu().pin_memory() for t in (h, y, logp_b, mask, cu, adv if has_bwd else logp_b[:1])]
         dev_in = [[torch.empty_like(t, device=dev) for t in host] for _ in range(2)]
         h2d = sum(t.numel() * t.element_size() for t in host)
         copy_stream = torch.cuda.Stream()
@@ -342,10 +353,11 @@ def run_ours(args):
                "sample": f"first {rows} packed tokens of the workload (one sequence slice): fp64 forward over "
                          f"V={V}, filter, backward; {secs:.1f} s"}
 
-    launches_per_step = 2 + 1 + 5  # forward + finalize; filter; select, gather, dZ, dH, dW (one chunk)
+    # forward + finalize; filter; select, gather, dZ, dH, dW (one row chunk)
+    launches_per_step = 2 + 1 + (5 if has_bwd else 0)
     if rank == 0:
         line = {
-            "metric": METRIC,
+            "metric": METRIC if has_bwd else METRIC_FWD,
             "value": value,
             "unit": "tokens/s",
             "n_gpus": world,
@@ -359,7 +371,8 @@ def run_ours(args):
             "data": "synthetic",
             "config": {"workload": spec.name, "tokens_per_step": N, "sequences": B, "d": d, "V": V,
                        "delta": delta, "kept_sequences": n_keep_seq, "kept_tokens": kept_rows,
-                       "l2": "inputs larger than L2 (hidden 1.1 GB, W 2.0 GB); no flush",
+                       "l2": (f"inputs larger than L2 (hidden {N * d * 2 / 1e9:.2f} GB, W {V * d * 2 / 1e9:.2f} GB); "
+                              "no flush") if (N + V) * d * 2 > 129e6 else "flush: none (inputs fit in L2)",
                        "parallelism": f"replicas x{world}"},
             "pct_of_bf16_peak": step_tflops / peak_tf,
             "step_tflops_algorithmic": step_tflops,
@@ -369,10 +382,10 @@ def run_ours(args):
             "gpu_launches": launches_per_step * args.steps,
             "roofline": {"bound": "tensor", "kernel": "forward (tcgen05 projection + online log-softmax)",
                          "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s", "frac": achieved / peak_tf,
-                         "peak_source": f"{peaks['source']} bf16 sustained", "traffic": traffic},
-            "roofline_backward": {"bound": "tensor", "achieved": flop_bwd / (t_bwd / 1e3) / 1e12,
-                                  "peak": peak_tf, "unit": "TFLOP/s",
-                                  "frac": flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf},
+                         "peak_source": f"{peaks['source']} bf16 {peak_kind}", "traffic": traffic},
+            "roofline_backward": None if not has_bwd else {
+                "bound": "tensor", "achieved": flop_bwd / (t_bwd / 1e3) / 1e12, "peak": peak_tf, "unit": "TFLOP/s",
+                "frac": flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf},
             "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)
@@ -470,7 +483,7 @@ def run_reference(args):
         return
     from paper_2606_04847_gb300 import workloads
 
-    spec = workloads.spec_for(CONFIG_ID)
+    spec = workloads.spec_for(args.config)
     wl = workloads.build(spec, "cuda" if torch.cuda.is_available() else "cpu")
     rows = args.ref_rows
     for _ in range(args.warmup):
@@ -481,7 +494,7 @@ def run_reference(args):
     value = rows * args.steps / total
     line = {
         "impl": "reference",
-        "metric": METRIC,
+        "metric": METRIC if spec.advantages else METRIC_FWD,
         "value": value,
         "unit": "tokens/s",
         "n_gpus": world,
@@ -508,6 +521,9 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, choices=[1, 2, 3, 4, 5], default=CONFIG_ID,
+                    help="workload: 5 (default) = 9B-class fwd+bwd; 1-4 = the forward-only workloads "
+                         "(step = forward + filter)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=384)
