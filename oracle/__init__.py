@@ -16,6 +16,8 @@ Modules
                      ratios (Eq. 4).
 ``oracle.grpo``      the masked GRPO clipped-surrogate loss (Eq. 5 / Eq. 17,
                      without the KL term) and its gradient.
+``oracle.advantage`` the PrimeEcho trajectory reward (Eq. 9-10) and the
+                     group-normalised advantage (Eq. 12 / Eq. 3).
 
 Every function names the passage it follows. Parity is pinned for every
 function by the ``-m "not gpu"`` tests in ``tests/test_oracle_*.py`` (brute
@@ -26,3 +28,4 @@ paper's worked example); none is "parity unpinned".
 from .logprobs import logits, token_logprobs, token_logprobs_bwd  # noqa: F401
 from .filter import seq_ratio_filter  # noqa: F401
 from .grpo import grpo_masked_loss  # noqa: F401
+from .advantage import group_advantage, prime_echo_reward  # noqa: F401
