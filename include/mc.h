@@ -237,6 +237,31 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
                               void* workspace, size_t workspace_bytes, mc_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * PrimeEcho trajectory reward and group-normalised advantage (§4.4.3).
+ *
+ * For trajectory i with per-turn scores s_{i,k} = scores[i*K + k - 1] and
+ * verification outcomes success[i*K + k - 1], over its n_turns[i] turns
+ * (clamped to [1, K]; turns beyond it did not run):
+ *   reward[i]    = alpha s_{i,1} + (1 - alpha) max_k s_{i,k}
+ *                  + beta1 1[success_{i,1}] + beta2 1[!success_{i,1} && success_{i,2}]   (Eq. 9-10)
+ *   advantage[i] = (reward[i] - mean_G) / (std_G + eps)                                  (Eq. 12)
+ * over groups of group_size consecutive trajectories (the G samples of one
+ * prompt); std_G is the sample standard deviation (divisor G - 1) and a group
+ * of one gets advantage 0. K = 1 with beta1 = beta2 = 0 is the single-turn
+ * GRPO advantage of Eq. 3 with reward[i] = s_{i,1}.
+ *
+ *   scores fp32 [T, K]; success uint8 [T, K]; n_turns int32 [T]
+ *   T a positive multiple of group_size; K >= 1; alpha in [0, 1];
+ *   beta1, beta2 >= 0; eps >= 0
+ *   reward fp32 [T] out or NULL; advantage fp32 [T] out (feed it to
+ *   mc_grpo_masked_loss as `advantages`)
+ * ------------------------------------------------------------------------ */
+mc_status mc_prime_echo_advantages(const float* scores, const uint8_t* success, const int32_t* n_turns,
+                                   int32_t T, int32_t K, int32_t group_size, float alpha, float beta1,
+                                   float beta2, float eps, float* reward, float* advantage,
+                                   mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Self-test of the bounded device wait used by every pipelined kernel: one
  * CTA waits on a shared-memory barrier that nothing ever signals, gives up
  * after `timeout_ns` nanoseconds (1e6 <= timeout_ns <= 1e10), sets

@@ -24,7 +24,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmc.so")
 
-SOURCES = ["mc_api.cu", "mc_fwd.cu", "mc_bwd.cu", "mc_filter.cu", "mc_loss.cu", "mc_noalloc.cu"]
+SOURCES = ["mc_api.cu", "mc_fwd.cu", "mc_bwd.cu", "mc_filter.cu", "mc_loss.cu", "mc_advantage.cu",
+           "mc_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
           "-I", INCLUDE, "-I", CSRC]

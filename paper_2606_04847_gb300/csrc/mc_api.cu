@@ -521,6 +521,37 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
   return MC_OK;
 }
 
+mc_status mc_prime_echo_advantages(const float* scores, const uint8_t* success, const int32_t* n_turns, int32_t T,
+                                   int32_t K, int32_t group_size, float alpha, float beta1, float beta2, float eps,
+                                   float* reward, float* advantage, mc_stream_t stream) {
+  if (T < 1 || K < 1 || group_size < 1 || T % group_size != 0) return MC_ERR_INVALID_ARG;
+  if (!(alpha >= 0.f && alpha <= 1.f) || !(beta1 >= 0.f) || !(beta2 >= 0.f) || !(eps >= 0.f) ||
+      !std::isfinite(beta1) || !std::isfinite(beta2) || !std::isfinite(eps))
+    return MC_ERR_INVALID_ARG;
+  if (!scores || !success || !n_turns || !advantage) return MC_ERR_INVALID_ARG;
+  if (!aligned(scores, 4) || !aligned(n_turns, 4) || !aligned(advantage, 4) || (reward && !aligned(reward, 4)))
+    return MC_ERR_INVALID_ARG;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  mc::AdvArgs a;
+  a.scores = scores;
+  a.success = success;
+  a.n_turns = n_turns;
+  a.n_groups = T / group_size;
+  a.G = group_size;
+  a.K = K;
+  a.alpha = alpha;
+  a.beta1 = beta1;
+  a.beta2 = beta2;
+  a.eps = eps;
+  a.reward = reward;
+  a.advantage = advantage;
+  cudaError_t e = mc::launch_group_advantage(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "advantage launch");
+  return MC_OK;
+}
+
 mc_status mc_selftest_bounded_wait(int32_t* dev_status, int64_t timeout_ns, mc_stream_t stream) {
   if (!dev_status || !aligned(dev_status, 4)) return MC_ERR_INVALID_ARG;
   if (timeout_ns < 1000000LL || timeout_ns > 10000000000LL) return MC_ERR_INVALID_ARG;

@@ -152,6 +152,18 @@ struct LossArgs {
 };
 cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream);
 
+struct AdvArgs {
+  const float* scores;     // [T, K]
+  const uint8_t* success;  // [T, K]
+  const int32_t* n_turns;  // [T]
+  long long n_groups;
+  int G, K;
+  float alpha, beta1, beta2, eps;
+  float* reward;           // [T] or null
+  float* advantage;        // [T]
+};
+cudaError_t launch_group_advantage(const AdvArgs& a, cudaStream_t stream);
+
 cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream);
 
 size_t gemm_smem_bytes();

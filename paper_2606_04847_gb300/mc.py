@@ -51,6 +51,7 @@ SIGNATURES = {
     "mc_seq_ratio_filter": (_I32, [_P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _P, _P, _P]),
     "mc_grpo_masked_loss_workspace_size": (_SZ, [_I32]),
     "mc_grpo_masked_loss": (_I32, [_P, _P, _P, _P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _SZ, _P]),
+    "mc_prime_echo_advantages": (_I32, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _F, _F, _P, _P, _P]),
     "mc_selftest_bounded_wait": (_I32, [_P, _I64, _P]),
 }
 
@@ -265,6 +266,25 @@ def grpo_masked_loss(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
                                    _ptr(out.get("seq_loss")), _ptr(out.get("n_clipped")), _ptr(workspace),
                                    workspace.numel(), _stream(stream))
     _check("mc_grpo_masked_loss", st)
+    return out
+
+
+def prime_echo_advantages(scores: torch.Tensor, success: torch.Tensor, n_turns: torch.Tensor, group_size: int,
+                          alpha: float = 0.75, beta1: float = 0.0, beta2: float = 0.0, eps: float = 1e-6, *,
+                          stream=None) -> dict:
+    """mc_prime_echo_advantages: {"reward" [T], "advantage" [T]} from per-turn scores [T, K]."""
+    _need(scores, "scores", torch.float32, 2)
+    _need(success, "success", torch.uint8, 2)
+    _need(n_turns, "n_turns", torch.int32, 1)
+    T, K = scores.shape
+    if success.shape != (T, K) or n_turns.shape[0] != T:
+        raise ValueError("shape mismatch")
+    out = {"reward": torch.empty(T, dtype=torch.float32, device=scores.device),
+           "advantage": torch.empty(T, dtype=torch.float32, device=scores.device)}
+    st = lib().mc_prime_echo_advantages(_ptr(scores), _ptr(success), _ptr(n_turns), T, K, int(group_size),
+                                        float(alpha), float(beta1), float(beta2), float(eps), _ptr(out["reward"]),
+                                        _ptr(out["advantage"]), _stream(stream))
+    _check("mc_prime_echo_advantages", st)
     return out
 
 

@@ -142,6 +142,19 @@ def test_loss_argument_checks(L):
     assert loss_call(L, ws_bytes=16) == WORKSPACE
 
 
+def adv_call(L, T=16, K=3, G=8, alpha=0.75, eps=1e-6, adv=FAKE):
+    return L.mc_prime_echo_advantages(FAKE, FAKE, FAKE, T, K, G, alpha, 0.5, 0.2, eps, None, adv, None)
+
+
+def test_advantage_argument_checks(L):
+    assert adv_call(L, T=10, G=8) == INVALID  # T not a multiple of the group size
+    assert adv_call(L, K=0) == INVALID
+    assert adv_call(L, G=0) == INVALID
+    assert adv_call(L, alpha=1.5) == INVALID
+    assert adv_call(L, eps=-1.0) == INVALID
+    assert adv_call(L, adv=None) == INVALID
+
+
 def test_selftest_argument_checks(L):
     assert L.mc_selftest_bounded_wait(None, 10 ** 8, None) == INVALID
     assert L.mc_selftest_bounded_wait(FAKE, 10, None) == INVALID
