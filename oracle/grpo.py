@@ -12,9 +12,14 @@ Paper passages followed
       s_{i,t} = min(rho A_i, clip(rho, 1 - eps_low, 1 + eps_high) A_i)
   summed over the tokens of every response, each response multiplied by its
   mask M_i, normalised by sum_i M_i L_i, negated:
-      L = -(1 / sum_i M_i L_i) sum_i sum_t s_{i,t} M_i.
-  The beta * KL(pi_theta || pi_ref) term of Eq. 17 is not part of this
-  function (the paper does not fix its estimator).
+      L = -(1 / sum_i M_i L_i) sum_i sum_t s_{i,t} M_i  +  beta KL.
+* The beta * KL(pi_theta || pi_ref) term of Eq. 5 / Eq. 17, estimated per
+  token from the sampled token's log-probs (the paper does not fix the
+  estimator; this is the non-negative per-token estimator used with GRPO):
+      k_t = pi_ref / pi_theta - log(pi_ref / pi_theta) - 1 = e^r - r - 1,
+      r = logp_ref_t - logp_policy_t,
+  averaged with the same mask and normaliser as the surrogate:
+      KL = (1 / sum_i M_i L_i) sum_i M_i sum_t k_t.
 
 Readings where the paper is silent
 ----------------------------------
@@ -43,12 +48,14 @@ def _mask(x, n):
 
 
 def grpo_masked_loss(logp_policy, logp_behaviour, loss_mask, cu_seqlens, advantages, keep,
-                     eps_low: float, eps_high: float):
-    """Masked GRPO loss (Eq. 17 without KL) and dL/dlogp_policy.
+                     eps_low: float, eps_high: float, logp_ref=None, beta: float = 0.0):
+    """Masked GRPO loss (Eq. 17) and dL/dlogp_policy.
 
     ``advantages`` [B] are the response-level advantages A_i (Eq. 3),
-    ``keep`` [B] the masks M_i (Eq. 21). Returns a dict with ``loss`` (float),
-    ``grad_logp`` [N], ``seq_loss`` [B] (each response's share of ``loss``),
+    ``keep`` [B] the masks M_i (Eq. 21); ``logp_ref`` [N] (optional) the
+    reference policy's log-probs for the beta * KL term. Returns a dict with
+    ``loss`` (float), ``grad_logp`` [N], ``seq_loss`` [B] (each response's
+    share of ``loss``), ``kl`` (the masked mean KL estimate, before beta),
     ``clipped`` [N] (bool: the clipped term was strictly smaller) and ``Z``.
     """
     lp = as_f64(logp_policy)
@@ -61,11 +68,13 @@ def grpo_masked_loss(logp_policy, logp_behaviour, loss_mask, cu_seqlens, advanta
     B = cu.shape[0] - 1
     L = np.array([m[cu[i]:cu[i + 1]].sum() for i in range(B)], dtype=np.float64)
     Z = float((M * L).sum())
+    lr = None if logp_ref is None else as_f64(logp_ref)
     grad = np.zeros(n)
     seq_loss = np.zeros(B)
+    kl_total = 0.0
     clipped = np.zeros(n, dtype=bool)
     if Z == 0.0:
-        return {"loss": 0.0, "grad_logp": grad, "seq_loss": seq_loss, "clipped": clipped, "Z": Z}
+        return {"loss": 0.0, "grad_logp": grad, "seq_loss": seq_loss, "kl": 0.0, "clipped": clipped, "Z": Z}
     for i in range(B):
         for t in range(cu[i], cu[i + 1]):
             if not m[t]:
@@ -79,4 +88,11 @@ def grpo_masked_loss(logp_policy, logp_behaviour, loss_mask, cu_seqlens, advanta
                 clipped[t] = True
             elif M[i] != 0.0:
                 grad[t] = -M[i] * rho * A[i] / Z
-    return {"loss": float(seq_loss.sum()), "grad_logp": grad, "seq_loss": seq_loss, "clipped": clipped, "Z": Z}
+            if lr is not None:
+                r = lr[t] - lp[t]
+                k = np.exp(r) - r - 1.0                                   # KL estimate per token
+                kl_total += M[i] * k / Z
+                seq_loss[i] += beta * M[i] * k / Z
+                grad[t] += beta * M[i] * (1.0 - np.exp(r)) / Z            # d k / d logp_policy
+    return {"loss": float(seq_loss.sum()), "grad_logp": grad, "seq_loss": seq_loss, "kl": float(kl_total),
+            "clipped": clipped, "Z": Z}

@@ -82,6 +82,36 @@ def test_masks_normaliser_and_all_dropped():
     assert sum(c["seq_loss"]) == pytest.approx(c["loss"], abs=1e-15)
 
 
+def test_kl_term_hand_computed_and_identity():
+    # one token, rho = 1 (so the surrogate is A = 0.5), reference prob twice the policy's:
+    # r = log 2, k = 2 - log 2 - 1; L = -0.5 + beta * k; dL/dlogp = -0.5 + beta * (1 - 2)
+    lp = np.array([-1.0])
+    lr = lp + np.log(2.0)
+    out = grpo_masked_loss(lp, lp, None, np.array([0, 1]), np.array([0.5]), np.array([1]), 0.2, 0.2,
+                           logp_ref=lr, beta=0.1)
+    k = 1.0 - np.log(2.0)
+    assert out["kl"] == pytest.approx(k, abs=1e-15)
+    assert out["loss"] == pytest.approx(-0.5 + 0.1 * k, abs=1e-15)
+    assert out["grad_logp"][0] == pytest.approx(-0.5 - 0.1, abs=1e-15)
+    # reference = policy: the KL term vanishes and changes nothing
+    lp2, lb2, mask, cu, A, keep = _random_case(4)
+    base = grpo_masked_loss(lp2, lb2, mask, cu, A, keep, 0.2, 0.28)
+    same = grpo_masked_loss(lp2, lb2, mask, cu, A, keep, 0.2, 0.28, logp_ref=lp2, beta=0.3)
+    assert same["kl"] == 0.0 and same["loss"] == pytest.approx(base["loss"], abs=1e-15)
+    np.testing.assert_allclose(same["grad_logp"], base["grad_logp"], atol=1e-15)
+
+
+def test_kl_estimate_is_nonnegative_and_masked():
+    rng = np.random.default_rng(5)
+    lp2, lb2, mask, cu, A, keep = _random_case(5)
+    lr = lp2 + rng.normal(0, 0.7, lp2.shape[0])
+    out = grpo_masked_loss(lp2, lb2, mask, cu, A, keep, 0.2, 0.28, logp_ref=lr, beta=0.05)
+    assert out["kl"] > 0.0
+    lr2 = lr.copy()
+    lr2[~mask.astype(bool)] += 5.0  # masked tokens never count
+    assert grpo_masked_loss(lp2, lb2, mask, cu, A, keep, 0.2, 0.28, logp_ref=lr2, beta=0.05)["kl"] == out["kl"]
+
+
 def _random_case(seed):
     rng = np.random.default_rng(seed)
     lens = [7, 1, 12, 5]
@@ -101,17 +131,23 @@ def _random_case(seed):
     return lp, lb, mask, cu, A, keep
 
 
-def test_gradient_central_differences():
+@pytest.mark.parametrize("with_kl", [False, True])
+def test_gradient_central_differences(with_kl):
     lp, lb, mask, cu, A, keep = _random_case(2)
-    out = grpo_masked_loss(lp, lb, mask, cu, A, keep, 0.2, 0.28)
+    lr = lp + np.random.default_rng(9).normal(0, 0.5, lp.shape[0]) if with_kl else None
+    beta = 0.2 if with_kl else 0.0
+
+    def loss(x):
+        return grpo_masked_loss(x, lb, mask, cu, A, keep, 0.2, 0.28, logp_ref=lr, beta=beta)["loss"]
+
+    out = grpo_masked_loss(lp, lb, mask, cu, A, keep, 0.2, 0.28, logp_ref=lr, beta=beta)
     eps = 1e-7
     fd = np.zeros_like(lp)
     for t in range(lp.shape[0]):
         p, q = lp.copy(), lp.copy()
         p[t] += eps
         q[t] -= eps
-        fd[t] = (grpo_masked_loss(p, lb, mask, cu, A, keep, 0.2, 0.28)["loss"]
-                 - grpo_masked_loss(q, lb, mask, cu, A, keep, 0.2, 0.28)["loss"]) / (2 * eps)
+        fd[t] = (loss(p) - loss(q)) / (2 * eps)
     np.testing.assert_allclose(out["grad_logp"], fd, atol=1e-8)
     assert out["clipped"].any() and (~out["clipped"] & mask.astype(bool)).any()
 
@@ -119,14 +155,17 @@ def test_gradient_central_differences():
 def test_gradient_matches_torch_autograd():
     torch = pytest.importorskip("torch")
     lp, lb, mask, cu, A, keep = _random_case(3)
-    out = grpo_masked_loss(lp, lb, mask, cu, A, keep, 0.2, 0.28)
+    lr = lp + np.random.default_rng(8).normal(0, 0.4, lp.shape[0])
+    out = grpo_masked_loss(lp, lb, mask, cu, A, keep, 0.2, 0.28, logp_ref=lr, beta=0.15)
     t_lp = torch.tensor(lp, requires_grad=True)
     seq = np.repeat(np.arange(len(A)), np.diff(cu))
     a_tok = torch.tensor(A[seq])
     w = torch.tensor(keep[seq] * mask, dtype=torch.float64)
     rho = torch.exp(t_lp - torch.tensor(lb))
     surr = torch.minimum(rho * a_tok, torch.clamp(rho, 0.8, 1.28) * a_tok)
-    loss = -(surr * w).sum() / w.sum()
+    r = torch.tensor(lr) - t_lp
+    kl = torch.exp(r) - r - 1.0
+    loss = -(surr * w).sum() / w.sum() + 0.15 * (kl * w).sum() / w.sum()
     loss.backward()
     assert out["loss"] == pytest.approx(loss.item(), abs=1e-14)
     np.testing.assert_allclose(out["grad_logp"], t_lp.grad.numpy(), atol=1e-14)
