@@ -209,21 +209,30 @@ mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behavi
  * L_i = n_tokens[i] (its loss-masked token count, as mc_seq_ratio_filter
  * returns it), over the tokens T_i of response i with loss_mask != 0:
  *   s_t          = min(rho_t A_i, clip(rho_t, 1 - eps_low, 1 + eps_high) A_i)   (Eq. 5)
- *   *loss        = -(1 / Z) sum_i M_i sum_{t in T_i} s_t,   Z = sum_i M_i L_i   (Eq. 17)
- *   grad_logp[t] = dL / dlogp_policy[t] = -M_i rho_t A_i / Z where the unclipped
- *                  term attains the minimum (ties included), else 0; 0 for
- *                  tokens with loss_mask == 0; everything 0 when Z == 0.
- * The beta * KL(pi_theta || pi_ref) term of Eq. 17 is not included (the paper
- * does not fix its estimator). grad_logp is the grad_logp argument of
- * mc_token_logprobs_bwd (dropped responses already carry zero gradient).
+ *   k_t          = e^r - r - 1,  r = logp_ref[t] - logp_policy[t]  (per-token
+ *                  estimate of KL(pi_theta || pi_ref); the paper does not fix
+ *                  the estimator, this is the non-negative one used with GRPO)
+ *   *kl          = (1 / Z) sum_i M_i sum_{t in T_i} k_t
+ *   *loss        = -(1 / Z) sum_i M_i sum_{t in T_i} s_t + beta * kl,
+ *                  Z = sum_i M_i L_i                                             (Eq. 17)
+ *   grad_logp[t] = dL / dlogp_policy[t] = (M_i / Z) (-rho_t A_i [where the
+ *                  unclipped term attains the minimum, ties included]
+ *                  + beta (1 - e^r)); 0 for tokens with loss_mask == 0;
+ *                  everything 0 when Z == 0.
+ * With logp_ref == NULL the KL term is absent (k_t = 0). grad_logp is the
+ * grad_logp argument of mc_token_logprobs_bwd (dropped responses already
+ * carry zero gradient).
  *
  *   advantages    fp32 [B]; keep uint8 [B]; n_tokens int32 [B]
  *   eps_low       in [0, 1); eps_high >= 0
+ *   logp_ref      fp32 [N] or NULL (reference-policy log-probs of the same tokens)
+ *   beta          KL weight >= 0 (ignored without logp_ref)
  *   loss          fp32 [1] out
  *   grad_logp     fp32 [N] out
  *   seq_loss      fp32 [B] out or NULL: response i's share of *loss
  *   n_clipped     int32 [1] out or NULL: tokens of kept responses whose clipped
  *                 term was strictly smaller
+ *   kl            fp32 [1] out or NULL
  *   workspace     >= mc_grpo_masked_loss_workspace_size(B) bytes, 256-byte aligned
  * Other arguments, layouts and error behaviour as for mc_seq_ratio_filter.
  * ------------------------------------------------------------------------ */
@@ -233,7 +242,8 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
                               const uint8_t* loss_mask, const int64_t* cu_seqlens,
                               const float* advantages, const uint8_t* keep, const int32_t* n_tokens,
                               int32_t B, int64_t N, float eps_low, float eps_high,
-                              float* loss, float* grad_logp, float* seq_loss, int32_t* n_clipped,
+                              const float* logp_ref, float beta,
+                              float* loss, float* grad_logp, float* seq_loss, int32_t* n_clipped, float* kl,
                               void* workspace, size_t workspace_bytes, mc_stream_t stream);
 
 /* ------------------------------------------------------------------------

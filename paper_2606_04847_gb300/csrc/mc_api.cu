@@ -471,17 +471,20 @@ mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behavi
 
 size_t mc_grpo_masked_loss_workspace_size(int32_t B) {
   if (B < 1) return 0;
-  return kStatusBytes + align_up(size_t(B) * sizeof(float), 256);
+  return kStatusBytes + 2 * align_up(size_t(B) * sizeof(float), 256);
 }
 
 mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behaviour, const uint8_t* loss_mask,
                               const int64_t* cu_seqlens, const float* advantages, const uint8_t* keep,
                               const int32_t* n_tokens, int32_t B, int64_t N, float eps_low, float eps_high,
-                              float* loss, float* grad_logp, float* seq_loss, int32_t* n_clipped, void* workspace,
-                              size_t workspace_bytes, mc_stream_t stream) {
+                              const float* logp_ref, float beta, float* loss, float* grad_logp, float* seq_loss,
+                              int32_t* n_clipped, float* kl, void* workspace, size_t workspace_bytes,
+                              mc_stream_t stream) {
   if (B < 1 || N < 0 || N >= (1LL << 40)) return MC_ERR_INVALID_ARG;
   if (!(eps_low >= 0.f && eps_low < 1.f) || !(eps_high >= 0.f) || !std::isfinite(eps_high))
     return MC_ERR_INVALID_ARG;
+  if (!(beta >= 0.f) || !std::isfinite(beta)) return MC_ERR_INVALID_ARG;
+  if ((logp_ref && !aligned(logp_ref, 4)) || (kl && !aligned(kl, 4))) return MC_ERR_INVALID_ARG;
   if (!cu_seqlens || !advantages || !keep || !n_tokens || !loss) return MC_ERR_INVALID_ARG;
   if (N > 0 && (!logp_policy || !logp_behaviour || !grad_logp)) return MC_ERR_INVALID_ARG;
   if (!aligned(cu_seqlens, 8) || !aligned(advantages, 4) || !aligned(n_tokens, 4) || !aligned(loss, 4) ||
@@ -507,14 +510,18 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
   a.N = N;
   a.eps_low = eps_low;
   a.eps_high = eps_high;
+  a.logp_ref = N > 0 ? logp_ref : nullptr;
+  a.beta = logp_ref ? beta : 0.f;
   a.loss = loss;
   a.grad_logp = grad_logp;
   a.seq_loss = seq_loss;
   a.n_clipped = n_clipped;
+  a.kl = kl;
   a.Z = reinterpret_cast<long long*>(ws);
   a.seq_share = reinterpret_cast<float*>(ws + kStatusBytes);
+  a.seq_kl = reinterpret_cast<float*>(ws + kStatusBytes + align_up(size_t(B) * sizeof(float), 256));
   a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && aligned(grad_logp, 16) &&
-             (!loss_mask || aligned(loss_mask, 4));
+             (!logp_ref || aligned(logp_ref, 16)) && (!loss_mask || aligned(loss_mask, 4));
   a.grid = 8 * sms;
   cudaError_t e = mc::launch_grpo_loss(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "GRPO loss launch");

@@ -141,12 +141,16 @@ struct LossArgs {
   int B;
   long long N;
   float eps_low, eps_high;
+  const float* logp_ref;  // null: no KL term
+  float beta;
   float* loss;
   float* grad_logp;
   float* seq_loss;
   int32_t* n_clipped;
+  float* kl;
   long long* Z;           // workspace
   float* seq_share;       // workspace [B]
+  float* seq_kl;          // workspace [B]
   int vec_ok;
   int grid;               // persistent CTAs (sequences are strided over them)
 };

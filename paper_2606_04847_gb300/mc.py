@@ -50,7 +50,8 @@ SIGNATURES = {
                                      _SZ, _P, _P]),
     "mc_seq_ratio_filter": (_I32, [_P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _P, _P, _P]),
     "mc_grpo_masked_loss_workspace_size": (_SZ, [_I32]),
-    "mc_grpo_masked_loss": (_I32, [_P, _P, _P, _P, _P, _P, _P, _I32, _I64, _F, _F, _P, _P, _P, _P, _P, _SZ, _P]),
+    "mc_grpo_masked_loss": (_I32, [_P, _P, _P, _P, _P, _P, _P, _I32, _I64, _F, _F, _P, _F, _P, _P, _P, _P, _P, _P,
+                                   _SZ, _P]),
     "mc_prime_echo_advantages": (_I32, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _F, _F, _P, _P, _P]),
     "mc_selftest_bounded_wait": (_I32, [_P, _I64, _P]),
 }
@@ -239,9 +240,12 @@ def seq_ratio_filter(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
 
 def grpo_masked_loss(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, loss_mask: Optional[torch.Tensor],
                      cu_seqlens: torch.Tensor, advantages: torch.Tensor, keep: torch.Tensor, n_tokens: torch.Tensor,
-                     eps_low: float, eps_high: float, *, out: Optional[dict] = None,
-                     workspace: Optional[torch.Tensor] = None, stream=None) -> dict:
-    """mc_grpo_masked_loss: {"loss" [1], "grad_logp" [N], "seq_loss" [B], "n_clipped" [1]}."""
+                     eps_low: float, eps_high: float, *, logp_ref: Optional[torch.Tensor] = None,
+                     beta: float = 0.0, out: Optional[dict] = None, workspace: Optional[torch.Tensor] = None,
+                     stream=None) -> dict:
+    """mc_grpo_masked_loss: {"loss" [1], "grad_logp" [N], "seq_loss" [B], "n_clipped" [1], "kl" [1]}."""
+    if logp_ref is not None:
+        _need(logp_ref, "logp_ref", torch.float32, 1)
     _need(logp_policy, "logp_policy", torch.float32, 1)
     _need(logp_behaviour, "logp_behaviour", torch.float32, 1)
     _need(cu_seqlens, "cu_seqlens", torch.int64, 1)
@@ -257,14 +261,15 @@ def grpo_masked_loss(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
         out = {"loss": torch.empty(1, dtype=torch.float32, device=dev),
                "grad_logp": torch.empty(N, dtype=torch.float32, device=dev),
                "seq_loss": torch.empty(B, dtype=torch.float32, device=dev),
-               "n_clipped": torch.empty(1, dtype=torch.int32, device=dev)}
+               "n_clipped": torch.empty(1, dtype=torch.int32, device=dev),
+               "kl": torch.empty(1, dtype=torch.float32, device=dev)}
     if workspace is None:
         workspace = torch.empty(lib().mc_grpo_masked_loss_workspace_size(B), dtype=torch.uint8, device=dev)
     st = lib().mc_grpo_masked_loss(_ptr(logp_policy), _ptr(logp_behaviour), _ptr(loss_mask), _ptr(cu_seqlens),
                                    _ptr(advantages), _ptr(keep), _ptr(n_tokens), B, N, float(eps_low),
-                                   float(eps_high), _ptr(out["loss"]), _ptr(out["grad_logp"]),
-                                   _ptr(out.get("seq_loss")), _ptr(out.get("n_clipped")), _ptr(workspace),
-                                   workspace.numel(), _stream(stream))
+                                   float(eps_high), _ptr(logp_ref), float(beta), _ptr(out["loss"]),
+                                   _ptr(out["grad_logp"]), _ptr(out.get("seq_loss")), _ptr(out.get("n_clipped")),
+                                   _ptr(out.get("kl")), _ptr(workspace), workspace.numel(), _stream(stream))
     _check("mc_grpo_masked_loss", st)
     return out
 

@@ -125,9 +125,10 @@ def test_filter_argument_checks(L):
     assert filt(L, cu=FAKE + 4) == INVALID  # int64 array not 8-byte aligned
 
 
-def loss_call(L, B=2, N=10, eps_low=0.2, eps_high=0.2, keep=FAKE, ws=FAKE, ws_bytes=1 << 20):
-    return L.mc_grpo_masked_loss(FAKE, FAKE, None, FAKE, FAKE, keep, FAKE, B, N, eps_low, eps_high, FAKE, FAKE,
-                                 None, None, ws, ws_bytes, None)
+def loss_call(L, B=2, N=10, eps_low=0.2, eps_high=0.2, keep=FAKE, ws=FAKE, ws_bytes=1 << 20, beta=0.0,
+              ref=None):
+    return L.mc_grpo_masked_loss(FAKE, FAKE, None, FAKE, FAKE, keep, FAKE, B, N, eps_low, eps_high, ref, beta,
+                                 FAKE, FAKE, None, None, None, ws, ws_bytes, None)
 
 
 def test_loss_argument_checks(L):
@@ -138,6 +139,9 @@ def test_loss_argument_checks(L):
     assert loss_call(L, eps_low=-0.1) == INVALID
     assert loss_call(L, eps_high=float("inf")) == INVALID
     assert loss_call(L, keep=None) == INVALID
+    assert loss_call(L, beta=-1.0) == INVALID
+    assert loss_call(L, beta=float("nan")) == INVALID
+    assert loss_call(L, ref=FAKE + 2) == INVALID  # misaligned reference log-probs
     assert loss_call(L, ws=None) == WORKSPACE
     assert loss_call(L, ws_bytes=16) == WORKSPACE
 
