@@ -124,6 +124,28 @@ def token_logprobs(hidden, w_vocab, targets, inv_temperature: float = 1.0,
     return {"logp": logp, "entropy": ent, "lse": lse}
 
 
+def logprob_state(hidden, w_shard, targets, v_begin: int, inv_temperature: float = 1.0):
+    """Softmax state of one vocabulary shard, columns [v_begin, v_begin + V_shard)
+    of a larger vocabulary (the rows w_shard of its LM head), per row t:
+        m = max_v z_{t,v},  s = sum_v exp(z - m),  t = sum_v exp(z - m)(z - m),
+        z_y = z_{t, y_t} if the shard holds y_t, else -inf.
+    Returns float64 [N, 4] = (m, s, t, z_y). Over a whole vocabulary,
+    lse = m + log s and entropy = log s - t / s (module docstring)."""
+    h = as_f64(hidden)
+    y = as_i64(targets)
+    z = (h @ as_f64(w_shard).T) * float(inv_temperature)
+    n, vs = z.shape
+    m = z.max(axis=1)
+    e = np.exp(z - m[:, None])
+    s = e.sum(axis=1)
+    t = (e * (z - m[:, None])).sum(axis=1)
+    local = y - int(v_begin)
+    own = (local >= 0) & (local < vs)
+    zy = np.full(n, -np.inf)
+    zy[own] = z[np.arange(n)[own], local[own]]
+    return np.stack([m, s, t, zy], axis=1)
+
+
 def token_logprobs_bwd(hidden, w_vocab, targets, grad_logp, grad_entropy=None,
                        inv_temperature: float = 1.0, return_dz: bool = False):
     """Closed-form gradients of L = sum_t g_t logp_t + sum_t gH_t H_t.

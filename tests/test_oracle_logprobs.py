@@ -156,6 +156,32 @@ def test_target_range_is_an_error():
         token_logprobs(np.ones((2, 4)), np.ones((3, 4)), np.array([-1, 0]))
 
 
+def test_shard_states_recombine_to_the_full_vocabulary():
+    """States of disjoint vocabulary shards, combined by rescaling to a common
+    max, give the full-vocabulary lse, entropy and target logit."""
+    from oracle.logprobs import logprob_state
+
+    rng = np.random.default_rng(9)
+    N, d, V = 7, 16, 50
+    h, w = _rand(rng, N, d), _rand(rng, V, d, scale=0.6)
+    y = rng.integers(0, V, N)
+    full = token_logprobs(h, w, y)
+    bounds = [0, 13, 14, 40, 50]  # includes a one-column shard
+    st = [logprob_state(h, w[a:b], y, a) for a, b in zip(bounds[:-1], bounds[1:])]
+    M = np.max([s[:, 0] for s in st], axis=0)
+    S = sum(s[:, 1] * np.exp(s[:, 0] - M) for s in st)
+    T = sum(np.exp(s[:, 0] - M) * (s[:, 2] + (s[:, 0] - M) * s[:, 1]) for s in st)
+    zy = np.max([s[:, 3] for s in st], axis=0)
+    np.testing.assert_allclose(M + np.log(S), full["lse"], atol=1e-12)
+    np.testing.assert_allclose(np.log(S) - T / S, full["entropy"], atol=1e-12)
+    np.testing.assert_allclose(zy - (M + np.log(S)), full["logp"], atol=1e-12)
+    # exactly one shard owns each target
+    owners = sum(np.isfinite(s[:, 3]).astype(int) for s in st)
+    np.testing.assert_array_equal(owners, 1)
+    for s in st:
+        assert np.all(s[:, 1] >= 1.0) and np.all(s[:, 2] <= 0.0)
+
+
 # ---------------------------------------------------------------- backward
 
 
