@@ -98,6 +98,37 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
                             int32_t* dev_status, mc_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Vocabulary-sharded forward: the building block of a tensor-parallel LM
+ * head (the paper trains its 27B model with tensor parallelism, §5.1).
+ *
+ * mc_token_logprob_state computes, for one slice of the vocabulary — the rows
+ * w_shard [V_shard, d] holding global ids [v_begin, v_begin + V_shard) — the
+ * softmax state of every row t, in natural units:
+ *   state[t] = (m, s, u, z_y):  m = max_v z[t, v],  s = sum_v exp(z - m),
+ *              u = sum_v exp(z - m) (z - m),
+ *              z_y = z[t, targets[t]] if the slice holds targets[t], else -inf
+ * (fp32 [N, 4], 16-byte aligned). targets are global ids. The workspace is
+ * mc_token_logprobs_workspace_size(N, d, V_shard) bytes.
+ *
+ * mc_merge_logprob_states combines P slice states (fp32 [P, N, 4], slice-major:
+ * the concatenation of the P state arrays, e.g. after an all-gather) into the
+ * full-vocabulary outputs of mc_token_logprobs:
+ *   M = max_p m_p, S = sum_p s_p e^(m_p - M), U = sum_p e^(m_p - M)(u_p + (m_p - M) s_p),
+ *   lse = M + log S, entropy = log S - U / S, logp = z_y - lse.
+ * The slices must partition the vocabulary; a row whose target no slice holds
+ * gets NaN outputs and sets MC_DEV_TARGET_RANGE.
+ * ------------------------------------------------------------------------ */
+mc_status mc_token_logprob_state(const void* hidden, const void* w_shard, const int32_t* targets,
+                                 int64_t N, int32_t d, int32_t V_shard, int32_t v_begin,
+                                 float inv_temperature, float* state,
+                                 void* workspace, size_t workspace_bytes,
+                                 int32_t* dev_status, mc_stream_t stream);
+
+mc_status mc_merge_logprob_states(const float* states, int32_t P, int64_t N,
+                                  float* logp, float* entropy, float* lse,
+                                  int32_t* dev_status, mc_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Forward for callers that cannot allocate device memory. (The paper has no
  * counterpart: this is a deployment variant of mc_token_logprobs.)
  *

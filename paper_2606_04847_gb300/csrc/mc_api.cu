@@ -241,16 +241,17 @@ size_t mc_token_logprobs_workspace_size(int64_t N, int32_t d, int32_t V) {
   return fwd_layout(N, V).total;
 }
 
-mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32_t* targets, int64_t N,
-                            int32_t d, int32_t V, float inv_temperature, float* logp, float* entropy,
-                            float* lse, void* workspace, size_t workspace_bytes, int32_t* dev_status,
-                            mc_stream_t stream) {
-  if (!valid_common(N, d, V, inv_temperature)) return MC_ERR_INVALID_ARG;
-  if (N == 0) return MC_OK;
-  if (!hidden || !w_vocab || !targets || !logp) return MC_ERR_INVALID_ARG;
-  if (!aligned(hidden, 16) || !aligned(w_vocab, 16) || !aligned(targets, 4) || !aligned(logp, 4) ||
-      (entropy && !aligned(entropy, 4)) || (lse && !aligned(lse, 4)) || (dev_status && !aligned(dev_status, 4)))
-    return MC_ERR_INVALID_ARG;
+}  // extern "C"
+
+namespace {
+
+// Queues the forward over the rows of W (a whole vocabulary, or a slice whose
+// row 0 is global id v_offset). Writes logp/entropy/lse, or with `state` the
+// slice state. Arguments are already validated.
+mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* targets, int64_t N, int32_t d,
+                        int32_t V, int32_t v_offset, float inv_temperature, float* logp, float* entropy, float* lse,
+                        float* state, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                        mc_stream_t stream) {
   const FwdLayout L = fwd_layout(N, V);
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < L.total) return MC_ERR_WORKSPACE;
   int sms = 0;
@@ -281,10 +282,59 @@ mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32
   a.grid = sms;
   a.timeout_ns = wait_timeout_ns();
   a.pair = use_pair_engine() ? 1 : 0;
+  a.v_offset = v_offset;
+  a.state = state;
   cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   e = mc::launch_forward(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "forward launch");
+  return MC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+mc_status mc_token_logprobs(const void* hidden, const void* w_vocab, const int32_t* targets, int64_t N,
+                            int32_t d, int32_t V, float inv_temperature, float* logp, float* entropy,
+                            float* lse, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                            mc_stream_t stream) {
+  if (!valid_common(N, d, V, inv_temperature)) return MC_ERR_INVALID_ARG;
+  if (N == 0) return MC_OK;
+  if (!hidden || !w_vocab || !targets || !logp) return MC_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(w_vocab, 16) || !aligned(targets, 4) || !aligned(logp, 4) ||
+      (entropy && !aligned(entropy, 4)) || (lse && !aligned(lse, 4)) || (dev_status && !aligned(dev_status, 4)))
+    return MC_ERR_INVALID_ARG;
+  return queue_forward(hidden, w_vocab, targets, N, d, V, 0, inv_temperature, logp, entropy, lse, nullptr,
+                       workspace, workspace_bytes, dev_status, stream);
+}
+
+mc_status mc_token_logprob_state(const void* hidden, const void* w_shard, const int32_t* targets, int64_t N,
+                                 int32_t d, int32_t V_shard, int32_t v_begin, float inv_temperature, float* state,
+                                 void* workspace, size_t workspace_bytes, int32_t* dev_status, mc_stream_t stream) {
+  if (!valid_common(N, d, V_shard, inv_temperature) || v_begin < 0) return MC_ERR_INVALID_ARG;
+  if (N == 0) return MC_OK;
+  if (!hidden || !w_shard || !targets || !state) return MC_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(w_shard, 16) || !aligned(targets, 4) || !aligned(state, 16) ||
+      (dev_status && !aligned(dev_status, 4)))
+    return MC_ERR_INVALID_ARG;
+  return queue_forward(hidden, w_shard, targets, N, d, V_shard, v_begin, inv_temperature, nullptr, nullptr, nullptr,
+                       state, workspace, workspace_bytes, dev_status, stream);
+}
+
+mc_status mc_merge_logprob_states(const float* states, int32_t P, int64_t N, float* logp, float* entropy, float* lse,
+                                  int32_t* dev_status, mc_stream_t stream) {
+  if (P < 1 || N < 0 || N >= (1LL << 31)) return MC_ERR_INVALID_ARG;
+  if (N == 0) return MC_OK;
+  if (!states || !logp || !aligned(states, 16) || !aligned(logp, 4) || (entropy && !aligned(entropy, 4)) ||
+      (lse && !aligned(lse, 4)) || (dev_status && !aligned(dev_status, 4)))
+    return MC_ERR_INVALID_ARG;
+  int sms = 0;
+  mc_status st = device_info(&sms);
+  if (st != MC_OK) return st;
+  cudaError_t e = mc::launch_merge_states(states, P, N, logp, entropy, lse, dev_status,
+                                          reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "state merge launch");
   return MC_OK;
 }
 

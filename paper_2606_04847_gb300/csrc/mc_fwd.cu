@@ -37,6 +37,7 @@ struct FwdEpi {
     float* zy;     // [n_pad]
     long long n_pad;
     int splits;
+    int v_offset;  // global id of column 0 (a vocabulary shard), 0 for the full vocabulary
   };
 
   float m, s0, s1, t0, t1;
@@ -47,7 +48,7 @@ struct FwdEpi {
   __device__ __forceinline__ void begin(const Params& p, long long row, int, int) {
     m = -INFINITY;
     s0 = s1 = t0 = t1 = 0.f;
-    y = row < p.N ? __ldg(p.targets + row) : -1;
+    y = row < p.N ? __ldg(p.targets + row) - p.v_offset : -1;  // column of the target in this W
   }
 
   // Online update with 32 values of which the first `nvalid` are real columns.
@@ -161,9 +162,89 @@ __global__ void fwd_finalize(const int32_t* __restrict__ targets, long long N, i
   if (lse) lse[row] = bad ? NAN : lse_v;
 }
 
+// Shard mode: the merged split partials of each row as a natural-unit state
+// (m, s, t, z_y) of this vocabulary slice; z_y = -inf when the slice does not
+// hold the row's target.
+__global__ void fwd_state_finalize(const int32_t* __restrict__ targets, long long N, int V, int v_offset,
+                                   int splits, long long n_pad, const float* __restrict__ part,
+                                   const float* __restrict__ zy, float4* __restrict__ state,
+                                   const int32_t* __restrict__ ws_status, int32_t* dev_status) {
+  const long long row = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (blockIdx.x == 0 && threadIdx.x == 0 && dev_status != nullptr && *ws_status != 0)
+    atomicOr(dev_status, *ws_status);
+  if (row >= N) return;
+  bool bad = (*ws_status & MC_DEV_TIMEOUT) != 0;
+  const long long plane = static_cast<long long>(splits) * n_pad;
+  float M = -INFINITY;
+  for (int k = 0; k < splits; ++k) {
+    const float mk = part[static_cast<long long>(k) * n_pad + row];
+    bad |= isnan(mk);
+    M = fmaxf(M, mk);
+  }
+  float S = 0.f, T = 0.f;
+  for (int k = 0; k < splits; ++k) {
+    const long long o = static_cast<long long>(k) * n_pad + row;
+    const float sk = part[plane + o];
+    if (!(sk > 0.f)) continue;
+    const float dm = part[o] - M;
+    const float r = exp2f(dm);
+    S = fmaf(sk, r, S);
+    T = fmaf(r, fmaf(dm, sk, part[2 * plane + o]), T);
+  }
+  const int local = targets[row] - v_offset;
+  const float zv = (local >= 0 && local < V) ? zy[row] : -INFINITY;
+  state[row] = bad ? make_float4(NAN, NAN, NAN, NAN) : make_float4(kLn2 * M, S, kLn2 * T, zv);
+}
+
+// Per row: combine the P slice states into the full-vocabulary log-sum-exp,
+// entropy and target log-prob (the same rescale-to-a-common-max rule as the
+// online update). A row whose target no slice holds gets NaN and sets
+// MC_DEV_TARGET_RANGE.
+__global__ void merge_states_kernel(const float4* __restrict__ states, int P, long long N, float* __restrict__ logp,
+                                    float* __restrict__ entropy, float* __restrict__ lse, int32_t* dev_status) {
+  const long long row = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (row >= N) return;
+  float M = -INFINITY, zv = -INFINITY;
+  bool bad = false;
+  for (int p = 0; p < P; ++p) {
+    const float4 s = states[static_cast<long long>(p) * N + row];
+    bad |= isnan(s.x);
+    M = fmaxf(M, s.x);
+    zv = fmaxf(zv, s.w);
+  }
+  float S = 0.f, T = 0.f;
+  for (int p = 0; p < P; ++p) {
+    const float4 s = states[static_cast<long long>(p) * N + row];
+    if (!(s.y > 0.f)) continue;
+    const float dm = s.x - M;
+    const float r = __expf(dm);
+    S = fmaf(s.y, r, S);
+    T = fmaf(r, fmaf(dm, s.y, s.z), T);
+  }
+  const bool no_target = !(zv > -INFINITY);
+  if (__any_sync(__activemask(), no_target) && dev_status != nullptr && (threadIdx.x & 31) == 0)
+    atomicOr(dev_status, MC_DEV_TARGET_RANGE);
+  bad |= no_target;
+  const float ls = logf(S);
+  const float lse_v = M + ls;
+  logp[row] = bad ? NAN : zv - lse_v;
+  if (entropy) entropy[row] = bad ? NAN : ls - T / S;
+  if (lse) lse[row] = bad ? NAN : lse_v;
+}
+
 }  // namespace
 
 size_t gemm_smem_bytes() { return GEMM_SMEM_BYTES; }
+
+cudaError_t launch_merge_states(const float* states, int P, long long N, float* logp, float* entropy, float* lse,
+                                int32_t* dev_status, cudaStream_t stream) {
+  if (N <= 0) return cudaSuccess;
+  const int threads = 256;
+  const long long blocks = (N + threads - 1) / threads;
+  merge_states_kernel<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
+      reinterpret_cast<const float4*>(states), P, N, logp, entropy, lse, dev_status);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   cudaError_t e;
@@ -183,6 +264,7 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   ep.zy = a.zy;
   ep.n_pad = a.n_pad;
   ep.splits = a.splits;
+  ep.v_offset = a.v_offset;
   if (a.pair) {
     e = run_gemm_pair<FwdEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
   } else {
@@ -198,9 +280,14 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int threads = 256;
   const long long blocks = (a.N + threads - 1) / threads;
-  fwd_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-      a.targets, a.N, a.V, a.splits, a.n_pad, a.part, a.zy, a.logp, a.entropy, a.lse, a.ws_status,
-      a.dev_status);
+  if (a.state != nullptr)
+    fwd_state_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
+        a.targets, a.N, a.V, a.v_offset, a.splits, a.n_pad, a.part, a.zy, reinterpret_cast<float4*>(a.state),
+        a.ws_status, a.dev_status);
+  else
+    fwd_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
+        a.targets, a.N, a.V, a.splits, a.n_pad, a.part, a.zy, a.logp, a.entropy, a.lse, a.ws_status,
+        a.dev_status);
   return cudaGetLastError();
 }
 

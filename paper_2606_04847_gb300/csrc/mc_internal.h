@@ -30,8 +30,12 @@ struct FwdArgs {
   int grid;
   uint64_t timeout_ns;
   int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
+  int v_offset;           // global vocabulary id of W's row 0 (shards); 0 otherwise
+  float* state;           // non-null: write the slice state [N, 4] instead of logp/entropy/lse
 };
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream);
+cudaError_t launch_merge_states(const float* states, int P, long long N, float* logp, float* entropy, float* lse,
+                                int32_t* dev_status, cudaStream_t stream);
 
 // Backward building blocks. Rows are first compacted on the device (idx[],
 // *count); every later stage takes its extent from *count.

@@ -45,6 +45,8 @@ SIGNATURES = {
     "mc_token_logprobs_workspace_size": (_SZ, [_I64, _I32, _I32]),
     "mc_token_logprobs": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _SZ, _P, _P]),
     "mc_token_logprobs_noalloc": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _P]),
+    "mc_token_logprob_state": (_I32, [_P, _P, _P, _I64, _I32, _I32, _I32, _F, _P, _P, _SZ, _P, _P]),
+    "mc_merge_logprob_states": (_I32, [_P, _I32, _I64, _P, _P, _P, _P, _P]),
     "mc_token_logprobs_bwd_workspace_size": (_SZ, [_I64, _I32, _I32, _I64]),
     "mc_token_logprobs_bwd": (_I32, [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _I32, _P,
                                      _SZ, _P, _P]),
@@ -146,6 +148,42 @@ def token_logprobs(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.T
                                  _ptr(out["logp"]), _ptr(out.get("entropy")), _ptr(out.get("lse")),
                                  _ptr(workspace), workspace.numel(), _ptr(dev_status), _stream(stream))
     _check("mc_token_logprobs", st)
+    return out
+
+
+def token_logprob_state(hidden: torch.Tensor, w_shard: torch.Tensor, targets: torch.Tensor, v_begin: int,
+                        inv_temperature: float = 1.0, *, state: Optional[torch.Tensor] = None,
+                        workspace: Optional[torch.Tensor] = None, dev_status: Optional[torch.Tensor] = None,
+                        stream=None) -> torch.Tensor:
+    """mc_token_logprob_state: the [N, 4] softmax state (m, s, u, z_y) of one vocabulary slice."""
+    _need(hidden, "hidden", torch.bfloat16, 2)
+    _need(w_shard, "w_shard", torch.bfloat16, 2)
+    _need(targets, "targets", torch.int32, 1)
+    N, d = hidden.shape
+    Vs = w_shard.shape[0]
+    if state is None:
+        state = torch.empty((N, 4), dtype=torch.float32, device=hidden.device)
+    if workspace is None:
+        workspace = torch.empty(max(forward_workspace_size(N, d, Vs), 256), dtype=torch.uint8, device=hidden.device)
+    st = lib().mc_token_logprob_state(_ptr(hidden), _ptr(w_shard), _ptr(targets), N, d, Vs, int(v_begin),
+                                      float(inv_temperature), _ptr(state), _ptr(workspace), workspace.numel(),
+                                      _ptr(dev_status), _stream(stream))
+    _check("mc_token_logprob_state", st)
+    return state
+
+
+def merge_logprob_states(states: torch.Tensor, *, out: Optional[dict] = None,
+                         dev_status: Optional[torch.Tensor] = None, stream=None) -> dict:
+    """mc_merge_logprob_states: {"logp", "entropy", "lse"} from slice states [P, N, 4]."""
+    _need(states, "states", torch.float32, 3)
+    P, N, four = states.shape
+    if four != 4:
+        raise ValueError("states must be [P, N, 4]")
+    if out is None:
+        out = {k: torch.empty(N, dtype=torch.float32, device=states.device) for k in ("logp", "entropy", "lse")}
+    st = lib().mc_merge_logprob_states(_ptr(states), P, N, _ptr(out["logp"]), _ptr(out.get("entropy")),
+                                       _ptr(out.get("lse")), _ptr(dev_status), _stream(stream))
+    _check("mc_merge_logprob_states", st)
     return out
 
 

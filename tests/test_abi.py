@@ -159,6 +159,19 @@ def test_advantage_argument_checks(L):
     assert adv_call(L, adv=None) == INVALID
 
 
+def test_shard_argument_checks(L):
+    def state(v_begin=0, st=FAKE, d=64):
+        return L.mc_token_logprob_state(FAKE, FAKE, FAKE, 16, d, 100, v_begin, 1.0, st, FAKE, 1 << 20, None, None)
+
+    assert state(v_begin=-1) == INVALID
+    assert state(st=None) == INVALID
+    assert state(st=FAKE + 4) == INVALID  # state rows are float4: 16-byte alignment
+    assert state(d=65) == INVALID
+    assert L.mc_merge_logprob_states(FAKE, 0, 16, FAKE, None, None, None, None) == INVALID
+    assert L.mc_merge_logprob_states(FAKE + 8, 2, 16, FAKE, None, None, None, None) == INVALID
+    assert L.mc_merge_logprob_states(FAKE, 2, 0, FAKE, None, None, None, None) == 0
+
+
 def test_selftest_argument_checks(L):
     assert L.mc_selftest_bounded_wait(None, 10 ** 8, None) == INVALID
     assert L.mc_selftest_bounded_wait(FAKE, 10, None) == INVALID
