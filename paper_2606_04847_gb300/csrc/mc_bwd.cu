@@ -13,7 +13,11 @@
 // and stores dZ as bf16 (a gradient, not the logits) to the workspace.
 // Stage 2: grad_hidden[idx[j]] = (dZ . W)[j]   (A = dZ K-major, B = W N-major)
 // Stage 3: grad_w (+)= dZ^T . Hc                (A = dZ M-major, B = Hc N-major)
-// Stages 2-3 are plain tcgen05 GEMMs of the same engine with store epilogues.
+// Stages 2-3 are plain tcgen05 GEMMs of the same engine with store epilogues,
+// one output tile per unit, tiles grouped so that a wave reads few operand
+// bytes (Schedule::n_group). Every epilogue store is evict-first (st.cs): no
+// output is read again before it has left L2, and the operand tiles that the
+// concurrent CTAs share stay resident.
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
@@ -190,7 +194,7 @@ struct DzEpi {
       if (vc + 32 <= p.V) {
         uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) d4[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+        for (int q = 0; q < 4; ++q) __stcs(d4 + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]));
       } else {
         const int n = p.V - vc;
         uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
@@ -232,8 +236,8 @@ struct StoreBf16Epi {
       uint4* d4 = reinterpret_cast<uint4*>(p.out + orow * p.ld + col);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        d4[q] = make_uint4(pack_bf16x2(x[8 * q + 0], x[8 * q + 1]), pack_bf16x2(x[8 * q + 2], x[8 * q + 3]),
-                           pack_bf16x2(x[8 * q + 4], x[8 * q + 5]), pack_bf16x2(x[8 * q + 6], x[8 * q + 7]));
+        __stcs(d4 + q, make_uint4(pack_bf16x2(x[8 * q + 0], x[8 * q + 1]), pack_bf16x2(x[8 * q + 2], x[8 * q + 3]),
+                                  pack_bf16x2(x[8 * q + 4], x[8 * q + 5]), pack_bf16x2(x[8 * q + 6], x[8 * q + 7])));
     }
   }
   __device__ __forceinline__ void end(const Params&, long long, int, int, bool) {}
@@ -268,13 +272,13 @@ struct StoreF32Epi {
         float4 v = kvalid ? make_float4(x[4 * q], x[4 * q + 1], x[4 * q + 2], x[4 * q + 3])
                           : make_float4(0.f, 0.f, 0.f, 0.f);
         if (p.accumulate) {
-          const float4 o = d4[q];
+          const float4 o = __ldcs(d4 + q);
           v.x += o.x;
           v.y += o.y;
           v.z += o.z;
           v.w += o.w;
         }
-        d4[q] = v;
+        __stcs(d4 + q, v);
       }
     }
   }
@@ -345,6 +349,24 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
                                               stream, a.pair);
 }
 
+// Tiles per group for a one-tile-per-unit long-K GEMM whose waves hold `conc`
+// units: the divisor b of n_tiles that minimises the operand extent one wave
+// streams, rb * conc / b (A rows) + BN * b (B columns), among those whose wave
+// still spans conc / b <= m_blocks row blocks. 0 = ungrouped.
+static int tile_group(int n_tiles, long long m_blocks, int conc, int rb) {
+  int best = 0;
+  double best_cost = double(rb) * conc / n_tiles + double(BN) * n_tiles;
+  for (int b = 1; b < n_tiles; ++b) {
+    if (n_tiles % b != 0 || static_cast<long long>(conc / b) > m_blocks) continue;
+    const double cost = double(rb) * conc / b + double(BN) * b;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = b;
+    }
+  }
+  return best;
+}
+
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   Schedule sch;
   const int rb = a.pair ? PAIR_BM : BM;
@@ -352,6 +374,7 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;  // one output tile per unit
   sch.k_blocks = (a.V + BK - 1) / BK;
+  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
@@ -373,6 +396,7 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;
   sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);
+  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;

@@ -80,9 +80,25 @@ struct Schedule {
   long long dyn_offset = 0;
   long long dyn_cap = 0;
   int dyn_mode = DYN_NONE;
+  // One-tile units only (splits == n_tiles): when 0 < n_group < n_tiles and
+  // n_group divides n_tiles, units are ordered (tile group, row block, tile in
+  // group), so the CTAs running at once cover ~grid/n_group row blocks x
+  // n_group tiles instead of ~grid/n_tiles x all tiles. A long-K GEMM re-reads
+  // both operands once per wave; this shape reads fewer bytes per wave.
+  int n_group = 0;
 
   __device__ __forceinline__ int units() const { return m_blocks * splits; }
   __device__ __forceinline__ void unit(int u, int& mb, int& split, int& t0, int& t1) const {
+    if (n_group > 0) {
+      const int per = m_blocks * n_group;
+      const int g = u / per;
+      const int r = u - g * per;
+      mb = r / n_group;
+      split = g * n_group + (r - mb * n_group);
+      t0 = split;
+      t1 = split + 1;
+      return;
+    }
     mb = u / splits;
     split = u - mb * splits;
     t0 = static_cast<int>((static_cast<long long>(split) * n_tiles) / splits);

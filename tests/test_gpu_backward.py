@@ -85,6 +85,16 @@ def test_vocab_tail_and_large_hidden():
     check(*setup(130, 5120, 300, seed=5))
 
 
+def test_single_entry_vocabulary_has_zero_gradient():
+    wl, g, ge = setup(129, 64, 1, seed=8)
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    fw = mc.token_logprobs(h, w, y)
+    out = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda())
+    torch.cuda.synchronize()
+    # p = 1 up to the rounding of exp2(z - lse): the gradient vanishes to ~1e-17
+    assert out["grad_hidden"].float().abs().max() < 1e-6 and out["grad_w"].abs().max() < 1e-6
+
+
 def test_peaked_softmax():
     check(*setup(256, 256, 2048, seed=6, w_scale=8.0))
 

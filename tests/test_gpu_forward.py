@@ -49,6 +49,16 @@ def test_ragged_shapes(N, d, V):
     run_and_compare(workloads.build(spec, "cpu"))
 
 
+@pytest.mark.parametrize("N,V", [(127, 1), (128, 31), (129, 33), (5, 257)])
+def test_tiny_vocabularies_and_block_edges(N, V):
+    """V = 1 (logp = 0, entropy = 0), V inside the first 32-column chunk, N on
+    both sides of a 128-row block."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=64, V=V)
+    out, ref = run_and_compare(workloads.build(spec, "cpu"))
+    if V == 1:
+        assert np.abs(np_(out["logp"])).max() < 1e-5 and np.abs(np_(out["entropy"])).max() < 1e-5
+
+
 def test_targets_at_vocab_edges_and_temperature():
     spec = workloads.spec_for(1, n_seqs=2, len_lo=150, len_hi=150, d=256, V=1000)
     wl = workloads.build(spec, "cpu")
