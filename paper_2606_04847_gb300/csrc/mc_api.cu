@@ -139,29 +139,30 @@ mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
   return MC_OK;
 }
 
-// Vocabulary tile ranges per 128-row block. Enough units to spread over the
-// SMs for small N, and at least 8 so the CTAs running together share few row
-// blocks (their hidden rows stay in L2) for large N. Within that range, the
-// count whose units leave the fewest CTAs idle in the last wave (ties: fewer
-// splits, so W is streamed fewer times).
-int choose_splits(long long m_blocks, int n_tiles, int sms) {
-  long long lo = ceil_div(2LL * sms, m_blocks);
-  if (lo < 8) lo = 8;
+// Vocabulary tile ranges per row block. A wave of `conc` concurrent units
+// streams W once and keeps its conc / s row blocks of hidden rows in L2, so
+// s is at least the count that holds those rows under kWaveRowBytes. Among
+// the counts allowed, the one with the shortest critical path in tiles,
+// waves(s) x ceil(n_tiles / s); counts within 0.5 % of the best resolve to
+// the fewest splits (fewest W streams).
+constexpr double kWaveRowBytes = 40.0 * (1 << 20);
+
+int choose_splits(long long m_blocks, int n_tiles, int conc, int rb, int d) {
+  long long lo = static_cast<long long>(std::ceil(double(conc) * rb * d * 2.0 / kWaveRowBytes));
+  if (lo < 1) lo = 1;
   long long hi = kMaxSplits;
   if (hi > n_tiles) hi = n_tiles;
   if (lo > hi) lo = hi;
-  long long best = lo;
-  double best_idle = 2.0;
+  double best_path = 0.0;
   for (long long s = lo; s <= hi; ++s) {
-    const long long units = m_blocks * s;
-    const long long slots = ceil_div(units, sms) * sms;
-    const double idle = static_cast<double>(slots - units) / static_cast<double>(slots);
-    if (idle < best_idle - 1e-9) {
-      best_idle = idle;
-      best = s;
-    }
+    const double path = double(ceil_div(m_blocks * s, conc)) * double(ceil_div(n_tiles, s));
+    if (s == lo || path < best_path) best_path = path;
   }
-  return static_cast<int>(best < 1 ? 1 : best);
+  for (long long s = lo; s <= hi; ++s) {
+    const double path = double(ceil_div(m_blocks * s, conc)) * double(ceil_div(n_tiles, s));
+    if (path <= best_path * 1.005) return static_cast<int>(s);
+  }
+  return static_cast<int>(hi);
 }
 
 int max_splits(int V) {
@@ -270,7 +271,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.d = d;
   a.V = V;
   a.inv_temperature = inv_temperature;
-  a.splits = choose_splits(m_blocks, n_tiles, concurrent_units(sms));
+  a.splits = choose_splits(m_blocks, n_tiles, concurrent_units(sms), row_block(), d);
   a.n_pad = L.n_pad;
   a.part = reinterpret_cast<float*>(ws + L.part_off);
   a.zy = reinterpret_cast<float*>(ws + L.zy_off);
@@ -435,7 +436,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.d = d;
     za.V = V;
     za.inv_temperature = inv_temperature;
-    za.splits = choose_splits(ceil_div(rows, row_block()), n_tiles, concurrent_units(sms));
+    za.splits = choose_splits(ceil_div(rows, row_block()), n_tiles, concurrent_units(sms), row_block(), d);
     za.dz = dz;
     za.ld = vp;
     za.ws_status = ws_status;
