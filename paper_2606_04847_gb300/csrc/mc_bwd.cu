@@ -14,8 +14,8 @@
 // Stage 2: grad_hidden[idx[j]] = (dZ . W)[j]   (A = dZ K-major, B = W N-major)
 // Stage 3: grad_w (+)= dZ^T . Hc                (A = dZ M-major, B = Hc N-major)
 // Stages 2-3 are plain tcgen05 GEMMs of the same engine with store epilogues,
-// one output tile per unit, tiles grouped so that a wave reads few operand
-// bytes (Schedule::n_group). Every epilogue store is evict-first (st.cs): no
+// one output tile per unit, 256-row tiles once K is long (TileCfg<2>) and
+// tiles grouped so that a wave reads few operand bytes (Schedule::n_group). Every epilogue store is evict-first (st.cs): no
 // output is read again before it has left L2, and the operand tiles that the
 // concurrent CTAs share stay resident.
 #include <cuda_bf16.h>
@@ -285,12 +285,12 @@ struct StoreF32Epi {
   __device__ __forceinline__ void end(const Params&, long long, int, int, bool) {}
 };
 
-template <class Epi, bool A_MN, bool B_MN>
+template <class Epi, bool A_MN, bool B_MN, int MS = 1>
 cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedule& sch,
                      const typename Epi::Params& ep, int grid_cap, uint64_t timeout_ns, int32_t* status,
                      cudaStream_t stream, int pair) {
   if (pair) return run_gemm_pair<Epi, A_MN, B_MN>(ta, tb, sch, ep, timeout_ns, status, stream);
-  auto kern = gemm_persistent<Epi, A_MN, B_MN>;
+  auto kern = gemm_persistent<Epi, A_MN, B_MN, MS>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(GEMM_SMEM_BYTES));
   if (e != cudaSuccess) return e;
@@ -367,13 +367,18 @@ static int tile_group(int n_tiles, long long m_blocks, int conc, int rb) {
   return best;
 }
 
+// K extent (in BK blocks) from which grad_hidden / grad_w use the wide
+// 256-row tile: the un-overlapped epilogue is then < 1 % of a unit.
+constexpr int kWideMinKBlocks = 256;
+
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   Schedule sch;
-  const int rb = a.pair ? PAIR_BM : BM;
+  sch.k_blocks = (a.V + BK - 1) / BK;
+  const bool wide = !a.pair && sch.k_blocks >= kWideMinKBlocks;
+  const int rb = a.pair ? PAIR_BM : (wide ? 2 * BM : BM);
   sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;  // one output tile per unit
-  sch.k_blocks = (a.V + BK - 1) / BK;
   sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
@@ -385,17 +390,21 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   ep.ld = a.d;
   ep.rows = a.rows;
   ep.cols = a.d;
+  if (wide)
+    return run_gemm<StoreBf16Epi, false, true, 2>(a.tm_dz, a.tm_w_mn, sch, ep, a.grid, a.timeout_ns,
+                                                  a.ws_status, stream, 0);
   return run_gemm<StoreBf16Epi, false, true>(a.tm_dz, a.tm_w_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
                                              stream, a.pair);
 }
 
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   Schedule sch;
-  const int rb = a.pair ? PAIR_BM : BM;
+  sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);  // host bound; the kernel reads the count
+  const bool wide = !a.pair && sch.k_blocks >= kWideMinKBlocks;
+  const int rb = a.pair ? PAIR_BM : (wide ? 2 * BM : BM);
   sch.m_blocks = (a.V + rb - 1) / rb;
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;
-  sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);
   sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
@@ -407,6 +416,9 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   ep.rows = a.V;
   ep.cols = a.d;
   ep.accumulate = a.accumulate;
+  if (wide)
+    return run_gemm<StoreF32Epi, true, true, 2>(a.tm_dz_mn, a.tm_h_mn, sch, ep, a.grid, a.timeout_ns,
+                                                a.ws_status, stream, 0);
   return run_gemm<StoreF32Epi, true, true>(a.tm_dz_mn, a.tm_h_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
                                            stream, a.pair);
 }

@@ -14,7 +14,8 @@
 //   warps 2-5     epilogue: warp w reads TMEM lanes 32*(w%4)..+31, one output
 //                 row per thread, 32 columns per tcgen05.ld
 // The two accumulators let the epilogue of tile j overlap the MMAs of tile
-// j+1. Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a] per
+// j+1 (or, with MS = 2, hold the two 128-row halves of one 256 x 256 tile:
+// see TileCfg). Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a] per
 // accumulator. Every wait is bounded (mbar_wait), and on the way out each
 // role drains what it has in flight (TMA loads, MMAs) before TMEM is freed.
 //
@@ -121,11 +122,30 @@ struct Schedule {
 // `k_nonempty` is false when a DYN_K extent is 0 (the accumulator is then
 // never written and must be read as zero).
 
-template <class Epi, bool A_MN, bool B_MN>
+// MS = row sub-blocks per tile. MS = 1: 128 x 256 tiles, 4 x 48 KB stages,
+// two tiles in flight in TMEM (the epilogue of one overlaps the MMAs of the
+// next). MS = 2 ("wide"): 256 x 256 tiles computed as two M = 128 MMAs that
+// share each B stage, 3 x 64 KB stages, both TMEM accumulators on the one
+// tile in flight. A wide tile streams ~29 % fewer operand bytes per output
+// from HBM and a third fewer from L2, for long-K GEMMs whose K loop dwarfs
+// the epilogue it no longer overlaps. Unit row blocks are then 256 rows.
+template <int MS>
+struct TileCfg {
+  static_assert(MS == 1 || MS == 2, "one or two 128-row sub-blocks");
+  static constexpr int TBM = BM * MS;
+  static constexpr int STAGES = MS == 1 ? NUM_STAGES : 3;
+  static constexpr int SBYTES = MS * A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int SLOTS = NUM_ACC / MS;  // tiles in flight in TMEM
+  static_assert(STAGES * SBYTES <= NUM_STAGES * STAGE_BYTES, "ring exceeds the SMEM budget");
+  static_assert(STAGES <= NUM_STAGES && SLOTS >= 1, "barrier arrays are sized for the narrow tile");
+};
+
+template <class Epi, bool A_MN, bool B_MN, int MS = 1>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const Schedule sch_in, const typename Epi::Params ep, const uint64_t timeout_ns,
                     int32_t* dev_status) {
+  using C = TileCfg<MS>;
   Schedule sch = sch_in;
   long long rows_eff = -1;
   bool k_nonempty = true;
@@ -133,7 +153,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     long long c = static_cast<long long>(*sch.dyn_count) - sch.dyn_offset;
     c = c < 0 ? 0 : (c > sch.dyn_cap ? sch.dyn_cap : c);
     if (sch.dyn_mode == DYN_ROWS) {
-      sch.m_blocks = static_cast<int>((c + BM - 1) / BM);
+      sch.m_blocks = static_cast<int>((c + C::TBM - 1) / C::TBM);
       rows_eff = c;
     } else if (sch.dyn_mode == DYN_K) {
       sch.k_blocks = static_cast<int>((c + BK - 1) / BK);
@@ -148,12 +168,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
   if (threadIdx.x == 0) {
 #pragma unroll
-    for (int s = 0; s < NUM_STAGES; ++s) {
+    for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&sh->full[s], 1);
       mbar_init(&sh->empty[s], 1);
     }
 #pragma unroll
-    for (int a = 0; a < NUM_ACC; ++a) {
+    for (int a = 0; a < C::SLOTS; ++a) {
       mbar_init(&sh->tfull[a], 1);
       mbar_init(&sh->tempty[a], NUM_EPI_WARPS);
     }
@@ -182,23 +202,27 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
         int mb, split, t0, t1;
         sch.unit(u, mb, split, t0, t1);
+        const int row0 = mb * C::TBM;
         for (int t = t0; t < t1 && ok; ++t) {
           for (int kb = 0; kb < sch.k_blocks; ++kb) {
-            const int s = static_cast<int>(it % NUM_STAGES);
-            const uint32_t ph = (it / NUM_STAGES) & 1u;
+            const int s = static_cast<int>(it % C::STAGES);
+            const uint32_t ph = (it / C::STAGES) & 1u;
             if (!mbar_wait(&sh->empty[s], ph ^ 1u, abort, timeout_ns, dev_status)) {
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(&sh->full[s], STAGE_BYTES);
-            uint8_t* a = smem + s * STAGE_BYTES;
-            uint8_t* b = a + A_STAGE_BYTES;
+            mbar_arrive_expect_tx(&sh->full[s], C::SBYTES);
+            uint8_t* a = smem + s * C::SBYTES;
+            uint8_t* b = a + MS * A_STAGE_BYTES;
+            // Sub-block j of A lands at a + j * A_STAGE_BYTES in both layouts.
             if (!A_MN) {
-              tma_load_2d(a, &tmA, &sh->full[s], kb * BK, mb * BM);
+#pragma unroll
+              for (int j = 0; j < MS; ++j)
+                tma_load_2d(a + j * A_STAGE_BYTES, &tmA, &sh->full[s], kb * BK, row0 + j * BM);
             } else {
 #pragma unroll
-              for (int j = 0; j < BM / 64; ++j)
-                tma_load_2d(a + j * MN_BOX_BYTES, &tmA, &sh->full[s], mb * BM + j * 64, kb * BK);
+              for (int j = 0; j < C::TBM / 64; ++j)
+                tma_load_2d(a + j * MN_BOX_BYTES, &tmA, &sh->full[s], row0 + j * 64, kb * BK);
             }
             if (!B_MN) {
               tma_load_2d(b, &tmB, &sh->full[s], kb * BK, t * BN);
@@ -212,9 +236,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
       }
       // Let every load this thread issued land before the CTA can exit.
-      const uint32_t last = it < NUM_STAGES ? it : NUM_STAGES;
+      const uint32_t last = it < C::STAGES ? it : C::STAGES;
       for (uint32_t j = it - last; j < it; ++j)
-        mbar_wait(&sh->full[j % NUM_STAGES], (j / NUM_STAGES) & 1u, nullptr, timeout_ns, dev_status);
+        mbar_wait(&sh->full[j % C::STAGES], (j / C::STAGES) & 1u, nullptr, timeout_ns, dev_status);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -226,37 +250,41 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         int mb, split, t0, t1;
         sch.unit(u, mb, split, t0, t1);
         for (int t = t0; t < t1 && ok; ++t) {
-          const uint32_t acc = tc & 1u;
-          const uint32_t aph = (tc >> 1) & 1u;
+          const uint32_t acc = tc % C::SLOTS;
+          const uint32_t aph = (tc / C::SLOTS) & 1u;
           if (!mbar_wait(&sh->tempty[acc], aph ^ 1u, abort, timeout_ns, dev_status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem + acc * BN;
+          const uint32_t d_tmem = tmem + acc * (MS * BN);
           for (int kb = 0; kb < sch.k_blocks; ++kb) {
-            const int s = static_cast<int>(it % NUM_STAGES);
-            const uint32_t ph = (it / NUM_STAGES) & 1u;
+            const int s = static_cast<int>(it % C::STAGES);
+            const uint32_t ph = (it / C::STAGES) & 1u;
             if (!mbar_wait(&sh->full[s], ph, abort, timeout_ns, dev_status)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t a_addr = smem_u32(smem + s * STAGE_BYTES);
-            const uint32_t b_addr = a_addr + A_STAGE_BYTES;
+            const uint32_t a_addr = smem_u32(smem + s * C::SBYTES);
+            const uint32_t b_addr = a_addr + MS * A_STAGE_BYTES;
 #pragma unroll
             for (int k = 0; k < BK / UMMA_K; ++k) {
-              const uint64_t adesc = A_MN ? smem_desc_sw128(a_addr + k * (UMMA_K * 128), MN_BOX_BYTES, 1024)
-                                          : smem_desc_sw128(a_addr + k * (UMMA_K * 2), 16, 1024);
               const uint64_t bdesc = B_MN ? smem_desc_sw128(b_addr + k * (UMMA_K * 128), MN_BOX_BYTES, 1024)
                                           : smem_desc_sw128(b_addr + k * (UMMA_K * 2), 16, 1024);
-              umma_bf16(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+              for (int j = 0; j < MS; ++j) {
+                const uint32_t aj = a_addr + j * A_STAGE_BYTES;
+                const uint64_t adesc = A_MN ? smem_desc_sw128(aj + k * (UMMA_K * 128), MN_BOX_BYTES, 1024)
+                                            : smem_desc_sw128(aj + k * (UMMA_K * 2), 16, 1024);
+                umma_bf16(d_tmem + j * BN, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+              }
             }
             umma_commit(&sh->empty[s]);  // frees the stage once these MMAs have read it
             ++it;
           }
           if (!ok) break;
-          umma_commit(&sh->tfull[acc]);  // accumulator ready for the epilogue
+          umma_commit(&sh->tfull[acc]);  // accumulator(s) ready for the epilogue
           ++tc;
         }
       }
@@ -270,17 +298,19 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int row_in_block = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t tc = 0;
-    Epi epi;
-    epi.setup(ep, rows_eff, k_nonempty);
+    Epi epi[MS];  // one output row per sub-block
+#pragma unroll
+    for (int j = 0; j < MS; ++j) epi[j].setup(ep, rows_eff, k_nonempty);
     bool ok = true;
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       int mb, split, t0, t1;
       sch.unit(u, mb, split, t0, t1);
-      const long long row = static_cast<long long>(mb) * BM + row_in_block;
-      epi.begin(ep, row, mb, split);
+      const long long row = static_cast<long long>(mb) * C::TBM + row_in_block;
+#pragma unroll
+      for (int j = 0; j < MS; ++j) epi[j].begin(ep, row + j * BM, mb, split);
       for (int t = t0; t < t1; ++t) {
-        const uint32_t acc = tc & 1u;
-        const uint32_t aph = (tc >> 1) & 1u;
+        const uint32_t acc = tc % C::SLOTS;
+        const uint32_t aph = (tc / C::SLOTS) & 1u;
         // Every lane polls; the warp proceeds only if all lanes saw the phase
         // complete, so the warp-collective tcgen05.ld below stays converged.
         const bool got = mbar_wait(&sh->tfull[acc], aph, abort, timeout_ns, dev_status);
@@ -289,13 +319,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           break;
         }
         tc_fence_after();
-        epi.tile(ep, row, t, tmem + acc * BN + lane_off);
+#pragma unroll
+        for (int j = 0; j < MS; ++j) epi[j].tile(ep, row + j * BM, t, tmem + (acc * MS + j) * BN + lane_off);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh->tempty[acc]);
         ++tc;
       }
-      epi.end(ep, row, mb, split, ok);
+#pragma unroll
+      for (int j = 0; j < MS; ++j) epi[j].end(ep, row + j * BM, mb, split, ok);
     }
   }
 

@@ -95,6 +95,29 @@ def test_single_entry_vocabulary_has_zero_gradient():
     assert out["grad_hidden"].float().abs().max() < 1e-6 and out["grad_w"].abs().max() < 1e-6
 
 
+def test_wide_tile_grad_hidden_long_vocabulary():
+    """K = V >= 256 k-blocks: grad_hidden runs 256-row tiles (600 rows =
+    2 blocks + 88, vocabulary tail of 33 columns)."""
+    check(*setup(600, 256, 16481, seed=10))
+
+
+def test_wide_tile_grad_w_many_rows_with_accumulate():
+    """K = rows >= 256 k-blocks: grad_w runs 256-row vocabulary tiles
+    (V = 700 = 2 blocks + 188) over 16,500 rows, accumulating."""
+    wl, g, ge = setup(16500, 128, 700, seed=11)
+    base = torch.randn(700, 128, generator=torch.Generator().manual_seed(12))
+    check(wl, g, ge, accumulate_base=base)
+
+
+def test_wide_tile_with_short_device_count():
+    """The host sizes grad_w for all 16,500 rows (wide tiles); the keep-mask
+    leaves ~1/3 of them, so the device-side K is far shorter."""
+    wl, g, _ = setup(16500, 128, 700, seed=13)
+    g[np.arange(16500) % 3 != 0] = 0.0
+    out, _ = check(wl, g, None)
+    assert torch.count_nonzero(out["grad_hidden"][1::3]) == 0
+
+
 def test_peaked_softmax():
     check(*setup(256, 256, 2048, seed=6, w_scale=8.0))
 
