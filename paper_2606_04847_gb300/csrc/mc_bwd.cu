@@ -15,9 +15,10 @@
 // Stage 3: grad_w (+)= dZ^T . Hc                (A = dZ M-major, B = Hc N-major)
 // Stages 2-3 are plain tcgen05 GEMMs of the same engine with store epilogues,
 // one output tile per unit, 256-row tiles once K is long (TileCfg<2>) and
-// tiles grouped so that a wave reads few operand bytes (Schedule::n_group). Every epilogue store is evict-first (st.cs): no
-// output is read again before it has left L2, and the operand tiles that the
-// concurrent CTAs share stay resident.
+// tiles grouped so that a wave reads few operand bytes (Schedule::n_group).
+// Every epilogue store is evict-first (st.cs): no output is read again
+// before it has left L2, and the operand tiles that the concurrent CTAs
+// share stay resident.
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"

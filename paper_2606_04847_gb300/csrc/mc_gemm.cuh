@@ -15,8 +15,8 @@
 //                 row per thread, 32 columns per tcgen05.ld
 // The two accumulators let the epilogue of tile j overlap the MMAs of tile
 // j+1 (or, with MS = 2, hold the two 128-row halves of one 256 x 256 tile:
-// see TileCfg). Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a] per
-// accumulator. Every wait is bounded (mbar_wait), and on the way out each
+// see TileCfg). Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a]
+// per accumulator. Every wait is bounded (mbar_wait), and on the way out each
 // role drains what it has in flight (TMA loads, MMAs) before TMEM is freed.
 //
 // Work decomposition: the M dimension is cut into BM-row blocks, the N
