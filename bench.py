@@ -347,7 +347,7 @@ def run_ours(args):
     # ---------------------------------------------------------------- CPU oracle baseline (rank 0, N = 1)
     cpu = None
     if world == 1 and not args.no_cpu:
-        rows = args.cpu_rows
+        rows = min(args.cpu_rows, N)  # the tiny configuration has fewer tokens than the sample
         secs = oracle_sample_step(wl, rows, delta)
         cpu = {"value": rows / secs, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
                "sample": f"first {rows} packed tokens of the workload (one sequence slice): fp64 forward over "
@@ -485,7 +485,7 @@ def run_reference(args):
 
     spec = workloads.spec_for(args.config)
     wl = workloads.build(spec, "cuda" if torch.cuda.is_available() else "cpu")
-    rows = args.ref_rows
+    rows = min(args.ref_rows, wl.N)
     for _ in range(args.warmup):
         oracle_sample_step(wl, rows, spec.delta)
     total = 0.0
