@@ -90,9 +90,17 @@ bool use_pair_engine() {
   return pair;
 }
 
-// Rows per scheduled row block, TMA box height of K-major B, and how many
-// units run at once, for the selected engine.
-int row_block() { return use_pair_engine() ? 256 : kBM; }
+// Projection launches (forward, dZ) of the one-CTA engine with at least this
+// many rows use 256-row tiles (TileCfg<2>: a third less operand traffic per
+// FLOP, 8 epilogue warps); fewer rows keep 128-row tiles so that small
+// launches still spread over the SMs.
+constexpr long long kWideMinRows = 4096;
+bool wide_rows(long long rows) { return !use_pair_engine() && rows >= kWideMinRows; }
+
+// Rows per scheduled row block of a projection launch over `rows` rows, TMA
+// box height of K-major B, and how many units run at once, for the selected
+// engine.
+int row_block(long long rows) { return (use_pair_engine() || wide_rows(rows)) ? 256 : kBM; }
 int b_box_rows() { return use_pair_engine() ? 128 : kBN; }
 int concurrent_units(int sms) { return use_pair_engine() ? sms / 2 : sms; }
 
@@ -264,14 +272,14 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   mc::FwdArgs a;
   if ((st = make_tmap(&a.tm_hidden, hidden, d, N, d, kBM)) != MC_OK) return st;
   if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, b_box_rows())) != MC_OK) return st;
-  const long long m_blocks = ceil_div(N, row_block());
+  const long long m_blocks = ceil_div(N, row_block(N));
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
   a.targets = targets;
   a.N = N;
   a.d = d;
   a.V = V;
   a.inv_temperature = inv_temperature;
-  a.splits = choose_splits(m_blocks, n_tiles, concurrent_units(sms), row_block(), d);
+  a.splits = choose_splits(m_blocks, n_tiles, concurrent_units(sms), row_block(N), d);
   a.n_pad = L.n_pad;
   a.part = reinterpret_cast<float*>(ws + L.part_off);
   a.zy = reinterpret_cast<float*>(ws + L.zy_off);
@@ -283,6 +291,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.grid = sms;
   a.timeout_ns = wait_timeout_ns();
   a.pair = use_pair_engine() ? 1 : 0;
+  a.wide = wide_rows(N) ? 1 : 0;
   a.v_offset = v_offset;
   a.state = state;
   cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);
@@ -436,13 +445,15 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.d = d;
     za.V = V;
     za.inv_temperature = inv_temperature;
-    za.splits = choose_splits(ceil_div(rows, row_block()), n_tiles, concurrent_units(sms), row_block(), d);
+    const int rb = row_block(rows);
+    za.splits = choose_splits(ceil_div(rows, rb), n_tiles, concurrent_units(sms), rb, d);
     za.dz = dz;
     za.ld = vp;
     za.ws_status = ws_status;
     za.grid = sms;
     za.timeout_ns = tmo;
     za.pair = use_pair_engine() ? 1 : 0;
+    za.wide = wide_rows(rows) ? 1 : 0;
     if ((e = mc::launch_dz(za, s)) != cudaSuccess) return cuda_fail(e, "dZ launch");
 
     mc::DhArgs ha;

@@ -298,7 +298,7 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
   const int units = sch.m_blocks * sch.splits;  // host upper bound; the kernel may find fewer
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, GEMM_THREADS, GEMM_SMEM_BYTES, stream>>>(ta, tb, sch, ep, timeout_ns, status);
+  kern<<<grid, TileCfg<MS>::THREADS, GEMM_SMEM_BYTES, stream>>>(ta, tb, sch, ep, timeout_ns, status);
   return cudaGetLastError();
 }
 
@@ -321,7 +321,7 @@ cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   Schedule sch;
-  const int rb = a.pair ? PAIR_BM : BM;
+  const int rb = a.pair ? PAIR_BM : (a.wide ? 2 * BM : BM);
   sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
@@ -343,6 +343,13 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   ep.inv_temp = a.inv_temperature;
   ep.dz = static_cast<__nv_bfloat16*>(a.dz);
   ep.ld = a.ld;
+  if (a.wide && !a.pair) {
+    if (a.grad_entropy != nullptr)
+      return run_gemm<DzEpi<true>, false, false, 2>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns,
+                                                    a.ws_status, stream, 0);
+    return run_gemm<DzEpi<false>, false, false, 2>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns,
+                                                   a.ws_status, stream, 0);
+  }
   if (a.grad_entropy != nullptr)
     return run_gemm<DzEpi<true>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
                                                stream, a.pair);

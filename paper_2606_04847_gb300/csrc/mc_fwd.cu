@@ -234,7 +234,18 @@ __global__ void merge_states_kernel(const float4* __restrict__ states, int P, lo
 
 }  // namespace
 
-size_t gemm_smem_bytes() { return GEMM_SMEM_BYTES; }
+template <int MS>
+cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdEpi::Params& ep, cudaStream_t stream) {
+  auto kern = gemm_persistent<FwdEpi, false, false, MS>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(GEMM_SMEM_BYTES));
+  if (e != cudaSuccess) return e;
+  const int units = sch.m_blocks * sch.splits;
+  const int grid = units < a.grid ? units : a.grid;
+  kern<<<grid, TileCfg<MS>::THREADS, GEMM_SMEM_BYTES, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns,
+                                                                 a.ws_status);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_merge_states(const float* states, int P, long long N, float* logp, float* entropy, float* lse,
                                 int32_t* dev_status, cudaStream_t stream) {
@@ -249,7 +260,7 @@ cudaError_t launch_merge_states(const float* states, int P, long long N, float* 
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   cudaError_t e;
   Schedule sch;
-  const int row_block = a.pair ? PAIR_BM : BM;
+  const int row_block = a.pair ? PAIR_BM : (a.wide ? 2 * BM : BM);
   sch.m_blocks = static_cast<int>((a.N + row_block - 1) / row_block);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
@@ -267,15 +278,10 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   ep.v_offset = a.v_offset;
   if (a.pair) {
     e = run_gemm_pair<FwdEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
+  } else if (a.wide) {
+    e = run_forward_gemm<2>(a, sch, ep, stream);
   } else {
-    auto kern = gemm_persistent<FwdEpi, false, false>;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(GEMM_SMEM_BYTES));
-    if (e != cudaSuccess) return e;
-    const int units = sch.m_blocks * sch.splits;
-    const int grid = units < a.grid ? units : a.grid;
-    kern<<<grid, GEMM_THREADS, GEMM_SMEM_BYTES, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns,
-                                                         a.ws_status);
-    e = cudaGetLastError();
+    e = run_forward_gemm<1>(a, sch, ep, stream);
   }
   if (e != cudaSuccess) return e;
   const int threads = 256;

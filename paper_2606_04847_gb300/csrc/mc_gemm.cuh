@@ -6,13 +6,14 @@
 // an online log-sum-exp / entropy update, the backward into dZ, the backward
 // GEMMs into plain stores.
 //
-// CTA = 6 warps, one CTA per SM (the SMEM ring takes ~194 KB):
+// CTA = 2 + 4 * MS warps, one CTA per SM (the SMEM ring takes ~194 KB):
 //   warp 0        TMA producer: loads A/B k-blocks (BK = 64) into a 4-stage ring
 //   warp 1        TMEM allocator + MMA issuer (one thread): 4 x tcgen05.mma
 //                 (M=128, N=256, K=16) per k-block into one of two TMEM
 //                 accumulators (2 x 256 fp32 columns = all 512 columns)
-//   warps 2-5     epilogue: warp w reads TMEM lanes 32*(w%4)..+31, one output
-//                 row per thread, 32 columns per tcgen05.ld
+//   warps 2..     epilogue (4 warps per 128-row sub-block): warp w reads TMEM
+//                 lanes 32*(w%4)..+31 of its sub-block, one output row per
+//                 thread, 32 columns per tcgen05.ld
 // The two accumulators let the epilogue of tile j overlap the MMAs of tile
 // j+1 (or, with MS = 2, hold the two 128-row halves of one 256 x 256 tile:
 // see TileCfg). Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a]
@@ -126,9 +127,11 @@ struct Schedule {
 // two tiles in flight in TMEM (the epilogue of one overlaps the MMAs of the
 // next). MS = 2 ("wide"): 256 x 256 tiles computed as two M = 128 MMAs that
 // share each B stage, 3 x 64 KB stages, both TMEM accumulators on the one
-// tile in flight. A wide tile streams ~29 % fewer operand bytes per output
-// from HBM and a third fewer from L2, for long-K GEMMs whose K loop dwarfs
-// the epilogue it no longer overlaps. Unit row blocks are then 256 rows.
+// tile in flight, and 8 epilogue warps that drain the two halves at once. A
+// wide tile streams ~29 % fewer operand bytes per output from HBM and a third
+// fewer from L2, and its ring covers longer operand latency; the epilogue no
+// longer overlaps the MMAs, which costs a GEMM little when its K loop is long
+// or its epilogue short. Unit row blocks are then 256 rows.
 template <int MS>
 struct TileCfg {
   static_assert(MS == 1 || MS == 2, "one or two 128-row sub-blocks");
@@ -136,12 +139,14 @@ struct TileCfg {
   static constexpr int STAGES = MS == 1 ? NUM_STAGES : 3;
   static constexpr int SBYTES = MS * A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr int SLOTS = NUM_ACC / MS;  // tiles in flight in TMEM
+  static constexpr int EPI_WARPS = NUM_EPI_WARPS * MS;  // 4 per 128-row sub-block
+  static constexpr int THREADS = 32 * (EPI_WARP_BEGIN + EPI_WARPS);
   static_assert(STAGES * SBYTES <= NUM_STAGES * STAGE_BYTES, "ring exceeds the SMEM budget");
   static_assert(STAGES <= NUM_STAGES && SLOTS >= 1, "barrier arrays are sized for the narrow tile");
 };
 
 template <class Epi, bool A_MN, bool B_MN, int MS = 1>
-__global__ void __launch_bounds__(GEMM_THREADS, 1)
+__global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const Schedule sch_in, const typename Epi::Params ep, const uint64_t timeout_ns,
                     int32_t* dev_status) {
@@ -175,7 +180,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 #pragma unroll
     for (int a = 0; a < C::SLOTS; ++a) {
       mbar_init(&sh->tfull[a], 1);
-      mbar_init(&sh->tempty[a], NUM_EPI_WARPS);
+      mbar_init(&sh->tempty[a], C::EPI_WARPS);
     }
     mbar_init(&sh->drain, 1);
     sh->abort = 0;
@@ -294,20 +299,21 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int quad = warp & 3;  // TMEM lane quadrant this warp may access
-    const int row_in_block = quad * 32 + lane;
+    // Warps 2.. in groups of four, group j draining row sub-block j; within a
+    // group, warp w may access TMEM lane quadrant w % 4 only.
+    const int sub = (warp - EPI_WARP_BEGIN) / NUM_EPI_WARPS;
+    const int quad = warp & 3;
+    const int row_in_tile = sub * BM + quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t tc = 0;
-    Epi epi[MS];  // one output row per sub-block
-#pragma unroll
-    for (int j = 0; j < MS; ++j) epi[j].setup(ep, rows_eff, k_nonempty);
+    Epi epi;
+    epi.setup(ep, rows_eff, k_nonempty);
     bool ok = true;
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       int mb, split, t0, t1;
       sch.unit(u, mb, split, t0, t1);
-      const long long row = static_cast<long long>(mb) * C::TBM + row_in_block;
-#pragma unroll
-      for (int j = 0; j < MS; ++j) epi[j].begin(ep, row + j * BM, mb, split);
+      const long long row = static_cast<long long>(mb) * C::TBM + row_in_tile;
+      epi.begin(ep, row, mb, split);
       for (int t = t0; t < t1; ++t) {
         const uint32_t acc = tc % C::SLOTS;
         const uint32_t aph = (tc / C::SLOTS) & 1u;
@@ -319,15 +325,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           break;
         }
         tc_fence_after();
-#pragma unroll
-        for (int j = 0; j < MS; ++j) epi[j].tile(ep, row + j * BM, t, tmem + (acc * MS + j) * BN + lane_off);
+        epi.tile(ep, row, t, tmem + (acc * MS + sub) * BN + lane_off);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh->tempty[acc]);
         ++tc;
       }
-#pragma unroll
-      for (int j = 0; j < MS; ++j) epi[j].end(ep, row + j * BM, mb, split, ok);
+      epi.end(ep, row, mb, split, ok);
     }
   }
 

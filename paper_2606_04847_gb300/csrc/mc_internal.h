@@ -30,6 +30,7 @@ struct FwdArgs {
   int grid;
   uint64_t timeout_ns;
   int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
+  int wide;               // one-CTA engine only: 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
   int v_offset;           // global vocabulary id of W's row 0 (shards); 0 otherwise
   float* state;           // non-null: write the slice state [N, 4] instead of logp/entropy/lse
 };
@@ -76,6 +77,7 @@ struct DzArgs {
   int grid;
   uint64_t timeout_ns;
   int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
+  int wide;               // one-CTA engine only: 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
 };
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream);
 
@@ -174,6 +176,5 @@ cudaError_t launch_group_advantage(const AdvArgs& a, cudaStream_t stream);
 
 cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream);
 
-size_t gemm_smem_bytes();
 
 }  // namespace mc

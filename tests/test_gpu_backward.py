@@ -95,6 +95,12 @@ def test_single_entry_vocabulary_has_zero_gradient():
     assert out["grad_hidden"].float().abs().max() < 1e-6 and out["grad_w"].abs().max() < 1e-6
 
 
+def test_wide_tile_dz_producer():
+    """>= 4096 kept rows: the dZ producer runs 256-row tiles (4500 rows =
+    17 blocks + 148), with the entropy term and temperature."""
+    check(*setup(4500, 128, 1500, seed=14), inv_temp=1.0 / 0.9)
+
+
 def test_wide_tile_grad_hidden_long_vocabulary():
     """K = V >= 256 k-blocks: grad_hidden runs 256-row tiles (600 rows =
     2 blocks + 88, vocabulary tail of 33 columns)."""

@@ -49,6 +49,14 @@ def test_ragged_shapes(N, d, V):
     run_and_compare(workloads.build(spec, "cpu"))
 
 
+@pytest.mark.parametrize("inv_temp", [1.0, 1.0 / 0.9])
+def test_wide_tiles_ragged(inv_temp):
+    """>= 4096 rows: 256-row tiles with 8 epilogue warps (4500 rows = 17
+    blocks + 148), a vocabulary tail of 184 columns."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=4500, len_hi=4500, d=256, V=3000)
+    run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
+
+
 @pytest.mark.parametrize("N,V", [(127, 1), (128, 31), (129, 33), (5, 257)])
 def test_tiny_vocabularies_and_block_edges(N, V):
     """V = 1 (logp = 0, entropy = 0), V inside the first 32-column chunk, N on

@@ -22,8 +22,9 @@ def run_shards(h, w, y, bounds, inv_temp=1.0):
     return states, mc.merge_logprob_states(states)
 
 
-def test_uneven_slices_match_unsharded_and_oracle():
-    spec = workloads.spec_for(1, n_seqs=1, len_lo=300, len_hi=300, d=256, V=4097)
+@pytest.mark.parametrize("N", [300, 4200])  # 128-row and 256-row tiles
+def test_uneven_slices_match_unsharded_and_oracle(N):
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=256, V=4097)
     wl = workloads.build(spec, "cpu")
     h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
     bounds = [0, 1000, 1001, 1100, 4097]
