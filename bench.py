@@ -183,6 +183,19 @@ def oracle_sample_step(wl, rows, delta):
     return time.perf_counter() - t0
 
 
+def _blas():
+    """BLAS library NumPy was built against, and its thread count (the oracle's matmuls)."""
+    import numpy as np
+
+    name = "unknown"
+    try:
+        name = np.__config__.CONFIG["Build Dependencies"]["blas"]["name"]
+    except (AttributeError, KeyError, TypeError):
+        pass
+    threads = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS") or str(_cores())
+    return f"{name}, {threads} threads"
+
+
 def _cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -349,7 +362,7 @@ def run_ours(args):
     if world == 1 and not args.no_cpu:
         rows = min(args.cpu_rows, N)  # the tiny configuration has fewer tokens than the sample
         secs = oracle_sample_step(wl, rows, delta)
-        cpu = {"value": rows / secs, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+        cpu = {"value": rows / secs, "unit": "tokens/s", "cores": _cores(), "kind": "oracle", "blas": _blas(),
                "sample": f"first {rows} packed tokens of the workload (one sequence slice): fp64 forward over "
                          f"V={V}, filter, backward; {secs:.1f} s"}
 
@@ -508,7 +521,7 @@ def run_reference(args):
         "data": "synthetic",
         "config": {"workload": spec.name, "tokens_per_step": rows, "d": spec.d, "V": spec.V,
                    "note": "each step: the oracle on the first packed tokens of the workload"},
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": _cores(), "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": _cores(), "kind": "oracle", "blas": _blas(),
                          "sample": f"{rows} tokens per step"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }

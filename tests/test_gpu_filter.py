@@ -58,7 +58,8 @@ def make(lens, gap_std=0.2, seed=0, mask_p=None, cancel=False):
     return lp.float(), lb, mask, cu
 
 
-@pytest.mark.parametrize("delta,delta_v", [(0.0, -1.0), (0.05, 0.05), (0.2, 0.2), (math.log(2), 0.1)])
+@pytest.mark.parametrize("delta,delta_v", [(0.0, -1.0), (0.02, 0.02), (0.05, 0.05), (0.1, 0.1), (0.2, 0.2),
+                                           (math.log(2), 0.1)])
 def test_config_shaped_sequences(delta, delta_v):
     lens = torch.randint(512, 8193, (32,), generator=torch.Generator().manual_seed(3)).tolist()
     compare(*make(lens, seed=1), delta, delta_v)
