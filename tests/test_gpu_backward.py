@@ -101,6 +101,13 @@ def test_wide_tile_dz_producer():
     check(*setup(4500, 128, 1500, seed=14), inv_temp=1.0 / 0.9)
 
 
+def test_row_chunks_across_the_wide_tile_threshold():
+    """A workspace for 4352-row chunks: 9000 rows run as 4352 + 4352 (dZ on
+    256-row tiles) + 296 (128-row tiles), grad_w accumulating over chunks."""
+    wl, g, ge = setup(9000, 128, 600, seed=15)
+    check(wl, g, ge, rows_per_chunk=4352)
+
+
 def test_wide_tile_grad_hidden_long_vocabulary():
     """K = V >= 256 k-blocks: grad_hidden runs 256-row tiles (600 rows =
     2 blocks + 88, vocabulary tail of 33 columns)."""
