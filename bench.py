@@ -158,6 +158,19 @@ def _max_over_ranks(x, world):
     return _reduce(x, world, "max")
 
 
+def dp_grad_w_allreduce(grad_w, world):
+    """The backward's one data-parallel exchange: each rank's grad_w [V, d] is
+    the gradient of its own batch; a DP trainer needs their sum before the
+    optimizer step, so every rank ends with the sum over ranks (NCCL on GPUs).
+    Forward, filter, loss and grad_hidden are per-sequence / per-row and need
+    no exchange. One rank: nothing to do."""
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.all_reduce(grad_w, op=dist.ReduceOp.SUM)
+    return grad_w
+
+
 # --------------------------------------------------------------------------- CPU oracle leg
 
 
@@ -284,6 +297,8 @@ def run_ours(args):
             else:
                 r = call(part, inputs, stream, flt)
                 flt = r if part == "filter" else flt
+        if has_bwd:
+            dp_grad_w_allreduce(gw, world)  # never captured: replayed graphs end at the backward
         if record:
             e[3].record(stream)
             ev["fwd"].append((e[0], e[1]))
@@ -443,7 +458,8 @@ def run_ours(args):
                              "inputs fit in L2: a 256 MB write flushes it before every timed step, outside the "
                              "step's CUDA events (value = summed step times; e2e not flushed)",
                        "cuda_graph": use_graph,
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": (f"dp x{world}: grad_w all-reduced over ranks every step (NCCL)"
+                                       if has_bwd and world > 1 else f"replicas x{world}")},
             "pct_of_bf16_peak": step_tflops / peak_tf,
             "step_tflops_algorithmic": step_tflops,
             "ms_by_call": {"forward": t_fwd, "filter": t_flt, "backward": t_bwd},
