@@ -175,15 +175,18 @@ mc_status mc_token_logprobs_noalloc(const void* hidden, const void* w_vocab, con
  * `row_keep` (uint8 [N], nullable = all kept) applies that gate, so
  * g[t] and gH[t] count only where row_keep[t] != 0 (pass the filter's
  * token_keep). Rows with a zero effective upstream gradient contribute
- * nothing: their grad_hidden rows are written as zero. The logits are recomputed per tile
- * on the tensor cores and never stored; dZ (a gradient) is staged in bf16 in
- * the workspace.
+ * nothing: their grad_hidden rows are written as zero. The logits are
+ * recomputed per tile on the tensor cores and never stored; dZ (a gradient)
+ * is staged in bf16 in the workspace.
  *
  *   lse, entropy  fp32 [N] from the forward (entropy may be NULL when gH is NULL)
  *   grad_logp     fp32 [N]; grad_entropy fp32 [N] or NULL
- *   workspace     >= mc_token_logprobs_bwd_workspace_size(N, d, V, 128) bytes;
- *                 more workspace lets the rows run in fewer, larger chunks
- *                 (mc_token_logprobs_bwd_workspace_size(N, d, V, N) = one chunk)
+ *   workspace     >= mc_token_logprobs_bwd_workspace_size(N, d, V, 256) bytes
+ *                 (chunks of 256 rows; rows_per_chunk rounds up to a multiple
+ *                 of 256); more workspace lets the rows run in fewer, larger
+ *                 chunks (mc_token_logprobs_bwd_workspace_size(N, d, V, N) =
+ *                 one chunk). The call uses as many rows per chunk as
+ *                 workspace_bytes holds.
  *   Other arguments as for the forward. A target outside [0, V) sets
  *   MC_DEV_TARGET_RANGE; that row's gradient terms are dropped.
  * ------------------------------------------------------------------------ */

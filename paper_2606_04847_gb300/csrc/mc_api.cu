@@ -205,7 +205,8 @@ FwdLayout fwd_layout(int64_t N, int32_t V) {
 long long v_pad(int32_t V) { return ceil_div(V, 64) * 64; }
 
 // Backward workspace: [status | count] header, selected-row indices, the
-// gathered hidden rows (zero-padded to 128 rows), then the dZ chunk buffer.
+// gathered hidden rows (zero-padded to a 256-row multiple), then the dZ chunk
+// buffer.
 struct BwdLayout {
   size_t status_off, count_off, idx_off, hc_off, fixed;
   long long n_pad;
