@@ -526,7 +526,7 @@ mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behavi
   a.token_keep = token_keep;
   a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && (!token_ratio || aligned(token_ratio, 16)) &&
              (!loss_mask || aligned(loss_mask, 4));
-  a.grid = 8 * sms;
+  a.grid = 16 * sms;
   cudaError_t e = mc::launch_filter(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "filter launch");
   return MC_OK;
@@ -585,7 +585,7 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
   a.seq_kl = reinterpret_cast<float*>(ws + kStatusBytes + align_up(size_t(B) * sizeof(float), 256));
   a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && aligned(grad_logp, 16) &&
              (!logp_ref || aligned(logp_ref, 16)) && (!loss_mask || aligned(loss_mask, 4));
-  a.grid = 8 * sms;
+  a.grid = 16 * sms;
   cudaError_t e = mc::launch_grpo_loss(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "GRPO loss launch");
   return MC_OK;

@@ -18,7 +18,7 @@ namespace mc {
 
 namespace {
 
-constexpr int kFilterThreads = 256;
+constexpr int kFilterThreads = 128;
 
 struct Acc {
   float s, a;
