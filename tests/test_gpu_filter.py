@@ -65,6 +65,20 @@ def test_config_shaped_sequences(delta, delta_v):
     compare(*make(lens, seed=1), delta, delta_v)
 
 
+@pytest.mark.parametrize("mask_p", [None, 0.8])
+def test_staged_chunks_odd_offsets_and_array_tail(mask_p):
+    """Sequences staged in 4096-token chunks: one starting at an odd offset
+    and spanning three chunks, an empty one, one of a single token, and an
+    array length (12,295) that is not a multiple of 16, so the last tokens
+    are past the last full 16 bytes; repeated calls agree bit for bit."""
+    lens = [5, 0, 1, 8995, 3294]
+    lp, lb, mask, cu = make(lens, seed=21, mask_p=mask_p)
+    a, _ = compare(lp, lb, mask, cu, 0.1, 0.1)
+    b = mc.seq_ratio_filter(lp.cuda(), lb.cuda(), None if mask is None else mask.cuda(), cu.cuda(), 0.1, 0.1)
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+
+
 def test_masks_odd_offsets_empty_and_length_one():
     lens = [1, 0, 3, 5, 7, 0, 1, 130, 1023, 4, 9]  # odd starts exercise the scalar head/tail
     compare(*make(lens, seed=2, mask_p=0.6), 0.1, 0.1)
