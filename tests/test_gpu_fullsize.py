@@ -78,6 +78,57 @@ def test_filter_full_size(config, cancel):
                        MASK_BAND, "keep_vanilla")
 
 
+def test_filter_full_size_first_turn_mask():
+    """27B-class multi-turn batch with the paper's first-turn-only loss mask
+    (only the first turn's response tokens count)."""
+    spec = workloads.spec_for(4, d=64, V=128)
+    wl = workloads.build(spec, "cpu", first_turn_only=True)
+    g = torch.Generator().manual_seed(44)
+    lp = -torch.empty(wl.N).exponential_(0.5, generator=g)
+    lb = (lp.double() + wl.gap.double()).float()
+    mask, delta = wl.loss_mask, spec.delta
+    out = mc.seq_ratio_filter(lp.cuda(), lb.cuda(), mask.cuda(), wl.cu_seqlens.cuda(), delta, delta)
+    ref = oracle.seq_ratio_filter(lp.numpy(), lb.numpy(), mask.numpy(), wl.cu_seqlens.numpy(),
+                                  float(np.float32(delta)), float(np.float32(delta)))
+    np.testing.assert_array_equal(np_(out["n_tokens"]), ref["n_tokens"])
+    assert_close_rel(np.exp(np_(out["abs_mean"])), np.exp(ref["abs_mean"]), TOL_RATIO, "e^A")
+    assert_masks_match(np_(out["keep"]), ref["keep"], ref["abs_mean"], delta, MASK_BAND, "keep")
+    seq = np.repeat(np.arange(wl.B), np.diff(wl.cu_seqlens.numpy()))
+    np.testing.assert_array_equal(np_(out["token_keep"]).astype(bool),
+                                  np_(out["keep"]).astype(bool)[seq] & mask.numpy().astype(bool))
+
+
+@pytest.mark.parametrize("config,first_turn", [(4, False), (4, True), (5, False)])
+def test_loss_full_size(config, first_turn):
+    """Masked GRPO loss with the beta * KL term (Eq. 17) on the configuration's
+    sequence lengths and loss mask (config 4: multi-turn, prompt tokens masked,
+    every turn or the first turn only), keep-mask from the filter, asymmetric
+    clip."""
+    spec = workloads.spec_for(config, d=64, V=128)  # shapes of the token arrays only
+    wl = workloads.build(spec, "cpu", first_turn_only=first_turn)
+    g = torch.Generator().manual_seed(40 + config)
+    lp = -torch.empty(wl.N).exponential_(0.5, generator=g)
+    lb = (lp.double() + wl.gap.double()).float()
+    lr = (lp.double() + torch.randn(wl.N, generator=g).double() * 0.1).float()
+    adv = torch.randn(wl.B, generator=g)
+    mask = wl.loss_mask
+    flt = mc.seq_ratio_filter(lp.cuda(), lb.cuda(), mask.cuda(), wl.cu_seqlens.cuda(), spec.delta)
+    out = mc.grpo_masked_loss(lp.cuda(), lb.cuda(), mask.cuda(), wl.cu_seqlens.cuda(), adv.cuda(), flt["keep"],
+                              flt["n_tokens"], 0.2, 0.28, logp_ref=lr.cuda(), beta=0.04)
+    torch.cuda.synchronize()
+    keep = np_(flt["keep"])
+    ref = oracle.grpo_masked_loss(lp.numpy(), lb.numpy(), mask.numpy(), wl.cu_seqlens.numpy(), adv.numpy(), keep,
+                                  float(np.float32(0.2)), float(np.float32(0.28)), logp_ref=lr.numpy(),
+                                  beta=float(np.float32(0.04)))
+    assert abs(out["loss"].item() - ref["loss"]) <= 2e-5, (out["loss"].item(), ref["loss"])
+    assert abs(out["kl"].item() - ref["kl"]) <= 2e-5, (out["kl"].item(), ref["kl"])
+    gr = ref["grad_logp"]
+    rho = np.exp(lp.double().numpy() - lb.double().numpy())
+    near = (np.abs(rho - 0.8) <= 1e-5) | (np.abs(rho - 1.28) <= 1.28e-5)
+    np.testing.assert_allclose(np_(out["grad_logp"])[~near], gr[~near], rtol=1e-5,
+                               atol=1e-6 * float(np.abs(gr).max(initial=0.0)))
+
+
 def test_backward_full_size_9b():
     spec = workloads.spec_for(5)
     wl = workloads.build(spec, "cuda")
