@@ -124,8 +124,8 @@ EncodeFn encode_fn() {
 
 // 2-D bf16 tensor [outer, inner] with row stride `stride_elems`, 128-byte
 // swizzled boxes of {64, box_outer}; out-of-range elements read as zero.
-mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_elems,
-                    uint32_t box_outer) {
+mc_status make_tmap_box(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_elems,
+                        uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle) {
   EncodeFn fn = encode_fn();
   if (fn == nullptr) {
     g_last_cuda_error = "cuTensorMapEncodeTiled not available from the driver";
@@ -133,10 +133,10 @@ mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
   }
   const cuuint64_t dims[2] = {inner, outer};
   const cuuint64_t strides[1] = {stride_elems * 2};
-  const cuuint32_t box[2] = {64, box_outer};
+  const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     char buf[128];
@@ -145,6 +145,13 @@ mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
     return MC_ERR_CUDA;
   }
   return MC_OK;
+}
+
+// Operand tiles of the GEMM engines: boxes 64 elements (128 bytes) wide,
+// 128-byte swizzle.
+mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_elems,
+                    uint32_t box_outer) {
+  return make_tmap_box(m, base, inner, outer, stride_elems, 64, box_outer, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 // Vocabulary tile ranges per row block. A wave of `conc` concurrent units
@@ -450,6 +457,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.splits = choose_splits(ceil_div(rows, rb), n_tiles, concurrent_units(sms), rb, d);
     za.dz = dz;
     za.ld = vp;
+    if ((st = make_tmap_box(&za.tm_dz_st, dz, V, rows, vp, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)) != MC_OK) return st;
     za.ws_status = ws_status;
     za.grid = sms;
     za.timeout_ns = tmo;

@@ -106,6 +106,7 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ H, int row_vec, con
 // ---------------------------------------------------------------- stage 1
 
 struct DzParams {
+  CUtensorMap tm_st;  // dz as {V, rows}, box {32 columns, 32 rows}, 64-byte swizzle: the staged stores
   const int32_t* targets;
   const float* lse;
   const float* entropy;
@@ -126,13 +127,32 @@ template <bool kEntropy>
 struct DzEpi {
   using Params = DzParams;
 
+  // Staged stores (one-CTA engine): each epilogue warp writes its 32 rows x
+  // 32 columns of bf16 into one of two 2 KB shared-memory buffers in the
+  // 64-byte swizzle (row r's 16-byte piece q at position q ^ ((r >> 1) & 3),
+  // conflict-free), and one lane stores the box with TMA: whole lines reach
+  // L2 instead of 32 scattered 16-byte pieces per warp store instruction.
+  // The tensor map's extent clips rows past the chunk and columns past V.
+  // Without a buffer (the CTA-pair engine) each thread stores its own row.
+  static constexpr int kStageBytes = 4096;
+
   long long rows_lim;
   float lse2, cg, cgh, hrow;
   int y;
   bool valid;
+  uint8_t* sbuf;
+  uint32_t nstore;
 
   __device__ __forceinline__ void setup(const Params& p, long long rows_eff, bool) {
     rows_lim = rows_eff >= 0 ? rows_eff : p.rows;
+    sbuf = nullptr;
+    nstore = 0;
+  }
+  __device__ __forceinline__ void stage(uint8_t* buf) { sbuf = buf; }
+  // The last stores must have completed before the CTA exits.
+  __device__ __forceinline__ void finish() {
+    if ((threadIdx.x & 31) == 0) bulk_wait_group_all();
+    __syncwarp();
   }
 
   __device__ __forceinline__ void begin(const Params& p, long long row, int, int) {
@@ -157,7 +177,8 @@ struct DzEpi {
       float x[32];
       tmem_ld32(taddr + c * 32, x);
       const int vc = v0 + c * 32;
-      if (vc >= p.V || row >= p.rows) continue;
+      if (vc >= p.V) continue;  // the same for the whole warp
+      if (sbuf == nullptr && row >= p.rows) continue;
       uint32_t w[16];
       if (valid) {
         const float nl = -lse2;
@@ -190,6 +211,25 @@ struct DzEpi {
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) w[i] = 0u;
+      }
+      if (sbuf != nullptr) {
+        const int lane = threadIdx.x & 31;
+        if (row - lane >= p.rows) continue;  // the warp's rows all lie past the chunk: nothing to store
+        uint8_t* buf = sbuf + (nstore & 1u) * 2048u;
+        if (lane == 0) bulk_wait_group_read<1>();  // the store that last used this buffer has read it
+        __syncwarp();
+        uint4* r4 = reinterpret_cast<uint4*>(buf + lane * 64);
+        const int sw = (lane >> 1) & 3;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) r4[q ^ sw] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+        fence_proxy_async_shared();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&p.tm_st, buf, vc, static_cast<int32_t>(row - lane));
+          bulk_commit_group();
+        }
+        ++nstore;
+        continue;
       }
       __nv_bfloat16* dst = p.dz + row * p.ld + vc;
       if (vc + 32 <= p.V) {
@@ -292,13 +332,13 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
                      cudaStream_t stream, int pair) {
   if (pair) return run_gemm_pair<Epi, A_MN, B_MN>(ta, tb, sch, ep, timeout_ns, status, stream);
   auto kern = gemm_persistent<Epi, A_MN, B_MN, MS>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(GEMM_SMEM_BYTES));
+  constexpr size_t smem = TileCfg<MS>::template smem_bytes<Epi>();
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int units = sch.m_blocks * sch.splits;  // host upper bound; the kernel may find fewer
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, TileCfg<MS>::THREADS, GEMM_SMEM_BYTES, stream>>>(ta, tb, sch, ep, timeout_ns, status);
+  kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(ta, tb, sch, ep, timeout_ns, status);
   return cudaGetLastError();
 }
 
@@ -343,6 +383,7 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   ep.inv_temp = a.inv_temperature;
   ep.dz = static_cast<__nv_bfloat16*>(a.dz);
   ep.ld = a.ld;
+  ep.tm_st = a.tm_dz_st;
   if (a.wide && !a.pair) {
     if (a.grad_entropy != nullptr)
       return run_gemm<DzEpi<true>, false, false, 2>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns,

@@ -237,13 +237,12 @@ __global__ void merge_states_kernel(const float4* __restrict__ states, int P, lo
 template <int MS>
 cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdEpi::Params& ep, cudaStream_t stream) {
   auto kern = gemm_persistent<FwdEpi, false, false, MS>;
-  cudaError_t e =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(GEMM_SMEM_BYTES));
+  constexpr size_t smem = TileCfg<MS>::template smem_bytes<FwdEpi>();
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int units = sch.m_blocks * sch.splits;
   const int grid = units < a.grid ? units : a.grid;
-  kern<<<grid, TileCfg<MS>::THREADS, GEMM_SMEM_BYTES, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns,
-                                                                 a.ws_status);
+  kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status);
   return cudaGetLastError();
 }
 

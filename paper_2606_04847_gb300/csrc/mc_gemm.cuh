@@ -37,6 +37,8 @@
 // {64 n, 64 k}. Out-of-range rows/columns are zero-filled by TMA.
 #pragma once
 
+#include <type_traits>
+
 #include "mc_ptx.cuh"
 
 namespace mc {
@@ -67,6 +69,19 @@ struct GemmShared {
 };
 
 constexpr size_t GEMM_SMEM_BYTES = size_t(NUM_STAGES) * STAGE_BYTES + sizeof(GemmShared) + 1024;
+
+// Epilogues may ask for shared memory of their own: `static constexpr int
+// kStageBytes` per epilogue warp (1024-byte aligned). The engine then calls
+// `epi.stage(buffer)` after setup and `epi.finish()` after the last unit.
+template <class E, class = void>
+struct EpiStage {
+  static constexpr int bytes = 0;
+};
+template <class E>
+struct EpiStage<E, std::void_t<decltype(E::kStageBytes)>> {
+  static constexpr int bytes = E::kStageBytes;
+};
+constexpr size_t kEpiStageOffset = (size_t(NUM_STAGES) * STAGE_BYTES + sizeof(GemmShared) + 1023) / 1024 * 1024;
 
 enum DynMode : int { DYN_NONE = 0, DYN_ROWS = 1, DYN_K = 2 };
 
@@ -141,6 +156,12 @@ struct TileCfg {
   static constexpr int SLOTS = NUM_ACC / MS;  // tiles in flight in TMEM
   static constexpr int EPI_WARPS = NUM_EPI_WARPS * MS;  // 4 per 128-row sub-block
   static constexpr int THREADS = 32 * (EPI_WARP_BEGIN + EPI_WARPS);
+  // Dynamic shared memory of the kernel running epilogue E.
+  template <class E>
+  static constexpr size_t smem_bytes() {
+    return EpiStage<E>::bytes > 0 ? kEpiStageOffset + size_t(EPI_WARPS) * EpiStage<E>::bytes + 1024
+                                  : GEMM_SMEM_BYTES;
+  }
   static_assert(STAGES * SBYTES <= NUM_STAGES * STAGE_BYTES, "ring exceeds the SMEM budget");
   static_assert(STAGES <= NUM_STAGES && SLOTS >= 1, "barrier arrays are sized for the narrow tile");
 };
@@ -148,9 +169,10 @@ struct TileCfg {
 template <class Epi, bool A_MN, bool B_MN, int MS = 1>
 __global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const Schedule sch_in, const typename Epi::Params ep, const uint64_t timeout_ns,
-                    int32_t* dev_status) {
+                    const Schedule sch_in, const __grid_constant__ typename Epi::Params ep,
+                    const uint64_t timeout_ns, int32_t* dev_status) {
   using C = TileCfg<MS>;
+  static_assert(C::template smem_bytes<Epi>() <= 227 * 1024, "shared memory of one CTA exceeded");
   Schedule sch = sch_in;
   long long rows_eff = -1;
   bool k_nonempty = true;
@@ -308,6 +330,8 @@ __global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
     uint32_t tc = 0;
     Epi epi;
     epi.setup(ep, rows_eff, k_nonempty);
+    if constexpr (EpiStage<Epi>::bytes > 0)
+      epi.stage(smem + kEpiStageOffset + (warp - EPI_WARP_BEGIN) * EpiStage<Epi>::bytes);
     bool ok = true;
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       int mb, split, t0, t1;
@@ -333,6 +357,7 @@ __global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
       }
       epi.end(ep, row, mb, split, ok);
     }
+    if constexpr (EpiStage<Epi>::bytes > 0) epi.finish();
   }
 
   tc_fence_before();

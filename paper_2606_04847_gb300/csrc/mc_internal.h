@@ -73,6 +73,7 @@ struct DzArgs {
   int splits;
   void* dz;               // bf16 [rows, ld]
   long long ld;
+  CUtensorMap tm_dz_st;   // dz {V, rows}, box {32, 32}, 64-byte swizzle (the epilogue's TMA stores)
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
