@@ -101,6 +101,12 @@ def test_wide_tile_dz_producer():
     check(*setup(4500, 128, 1500, seed=14), inv_temp=1.0 / 0.9)
 
 
+def test_wide_tile_dz_27b_hidden_size():
+    """256-row dZ tiles at d = 5120 (80 k-blocks per tile), 4500 rows (a
+    ragged last 32-row store box), V = 700 (a 28-column last store box)."""
+    check(*setup(4500, 5120, 700, seed=16))
+
+
 def test_row_chunks_across_the_wide_tile_threshold():
     """A workspace for 4352-row chunks: 9000 rows run as 4352 + 4352 (dZ on
     256-row tiles) + 296 (128-row tiles), grad_w accumulating over chunks."""
