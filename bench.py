@@ -196,6 +196,26 @@ def oracle_sample_step(wl, rows, delta):
     return time.perf_counter() - t0
 
 
+def _l2_persisting_limit():
+    """Read-only: the L2 set-aside for persisting accesses that this context
+    sees (cudaDeviceGetLimit; None when the runtime cannot be found). Part of
+    the L2 is then unavailable to ordinary accesses, which changes the
+    forward's DRAM traffic (W re-reads per wave) though not its speed."""
+    import ctypes
+    import glob
+
+    for path in (glob.glob(os.path.join(os.path.dirname(torch.__file__), "lib", "libcudart.so*")) +
+                 glob.glob("/usr/local/cuda/lib64/libcudart.so*")):
+        try:
+            rt = ctypes.CDLL(path)
+            v = ctypes.c_size_t(0)
+            if rt.cudaDeviceGetLimit(ctypes.byref(v), 6) == 0:  # cudaLimitPersistingL2CacheSize
+                return int(v.value)
+        except OSError:
+            continue
+    return None
+
+
 def _blas():
     """BLAS library NumPy was built against, and its thread count (the oracle's matmuls)."""
     import numpy as np
@@ -458,6 +478,7 @@ def run_ours(args):
                              "inputs fit in L2: a 256 MB write flushes it before every timed step, outside the "
                              "step's CUDA events (value = summed step times; e2e not flushed)",
                        "cuda_graph": use_graph,
+                       "l2_persisting_limit_bytes": _l2_persisting_limit(),
                        "parallelism": (f"dp x{world}: grad_w all-reduced over ranks every step (NCCL)"
                                        if has_bwd and world > 1 else f"replicas x{world}")},
             "pct_of_bf16_peak": step_tflops / peak_tf,
@@ -468,7 +489,9 @@ def run_ours(args):
             "gpu_launches": launches_per_step * args.steps,
             "roofline": {"bound": "tensor", "kernel": "forward (tcgen05 projection + online log-softmax)",
                          "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s", "frac": achieved / peak_tf,
-                         "peak_source": f"{peaks['source']} bf16 {peak_kind}", "traffic": traffic},
+                         "peak_source": f"{peaks['source']} bf16 {peak_kind}", "traffic": traffic,
+                         "traffic_source": "ncu single-pass capture of the full launch (profiles/fwd_kernel_traffic.json)"
+                         if traffic is not None else None},
             "roofline_backward": None if not has_bwd else {
                 "bound": "tensor", "achieved": flop_bwd / (t_bwd / 1e3) / 1e12, "peak": peak_tf, "unit": "TFLOP/s",
                 "frac": flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf,
