@@ -296,7 +296,8 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
  *
  *   scores fp32 [T, K]; success uint8 [T, K]; n_turns int32 [T]
  *   T a positive multiple of group_size; K >= 1; alpha in [0, 1];
- *   beta1, beta2 >= 0; eps >= 0
+ *   beta1, beta2 >= 0 (the paper sets beta1 > beta2 >= 0 so that earlier
+ *   success earns more; the library does not require the order); eps >= 0
  *   reward fp32 [T] out or NULL; advantage fp32 [T] out (feed it to
  *   mc_grpo_masked_loss as `advantages`)
  * ------------------------------------------------------------------------ */

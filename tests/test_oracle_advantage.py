@@ -34,6 +34,25 @@ def test_early_success_bonus_cases():
     assert R1[0] == 0.0
 
 
+def test_earlier_success_never_earns_less():
+    """Eq. 10 with beta1 > beta2 >= 0 (the paper's condition): among
+    trajectories with the same per-turn scores that succeed, succeeding at
+    turn 1 earns at least as much as first succeeding at turn 2, which earns
+    at least as much as first succeeding later."""
+    rng = np.random.default_rng(7)
+    for _ in range(200):
+        K = int(rng.integers(3, 6))
+        scores = rng.uniform(-1.0, 2.0, size=(1, K)).repeat(3, axis=0)
+        ok = np.zeros((3, K), dtype=bool)
+        ok[0, 0] = True                      # first success at turn 1
+        ok[1, 1] = True                      # first success at turn 2
+        ok[2, int(rng.integers(2, K))] = True  # first success later
+        b2 = float(rng.uniform(0.0, 1.0))
+        b1 = b2 + float(rng.uniform(1e-3, 1.0))
+        R = prime_echo_reward(scores, ok, np.full(3, K), float(rng.uniform(0, 1)), b1, b2)
+        assert R[0] > R[1] >= R[2]
+
+
 def test_hand_computed_reward():
     # alpha = 0.75, scores (-0.5, 0.25, 1.0) over 3 turns, success at turn 3 only:
     # 0.75 * -0.5 + 0.25 * 1.0 + 0 = -0.125
