@@ -550,6 +550,100 @@ def run_stream(args):
     print(json.dumps(res), flush=True)
 
 
+def _time_calls(fn, launches):
+    fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(launches):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / launches
+
+
+def run_next(args):
+    """Measurements of the rows beyond the main path (CUDA events over
+    --launches calls each), one JSON line:
+    * the masked GRPO loss with the beta * KL term (reference log-probs) on
+      64M tokens in 16,384 sequences: HBM GB/s for 4 + 4 + 4 + 1 B read and
+      4 B written per token;
+    * the vocabulary-sharded forward on the 9B-class fwd+bwd tokens: W in 4
+      slices (a 4-way tensor-parallel LM head run in one process), TFLOP/s of
+      2NdV over the 4 slice calls, and the merge's HBM GB/s (16 B per slice
+      read + 12 B written per token);
+    * the PrimeEcho reward and group advantage: the paper's batch (64
+      prompts x groups of 8 = 512 trajectories, 4 turns: launch-bound) and 2^24."""
+    from paper_2606_04847_gb300 import build as mcbuild
+    from paper_2606_04847_gb300 import mc, workloads
+
+    torch.cuda.set_device(0)
+    if not os.path.exists(mc.lib_path()):
+        mcbuild.build()
+    peaks = _peaks()
+    res = {"case": "next", "launches": args.launches, "peak_source": peaks["source"]}
+
+    # masked GRPO loss + beta * KL
+    N, B = 64 * 1024 * 1024, 16384
+    g = torch.Generator(device="cuda").manual_seed(0)
+    lp = -torch.rand(N, generator=g, device="cuda") * 8
+    lb = lp + torch.randn(N, generator=g, device="cuda") * 0.2
+    lr = lp + torch.randn(N, generator=g, device="cuda") * 0.1
+    mask = (torch.rand(N, generator=g, device="cuda") < 0.9).to(torch.uint8)
+    cu = torch.linspace(0, N, B + 1, device="cuda").round().to(torch.int64)
+    adv = torch.randn(B, generator=g, device="cuda")
+    flt = mc.seq_ratio_filter(lp, lb, mask, cu, 0.2, 0.2)
+    out = mc.grpo_masked_loss(lp, lb, mask, cu, adv, flt["keep"], flt["n_tokens"], 0.2, 0.28, logp_ref=lr, beta=0.04)
+    ms = _time_calls(lambda: mc.grpo_masked_loss(lp, lb, mask, cu, adv, flt["keep"], flt["n_tokens"], 0.2, 0.28,
+                                                 logp_ref=lr, beta=0.04, out=out), args.launches)
+    gbs = 17 * N / (ms / 1e3) / 1e9
+    res["loss_kl"] = {"tokens": N, "ms": ms, "bytes_per_token": 17, "achieved_gbs": gbs,
+                      "frac": gbs / peaks["hbm_gbs"], "peak_gbs": peaks["hbm_gbs"]}
+    del lp, lb, lr, mask, cu, adv, flt, out
+    torch.cuda.empty_cache()
+
+    # vocabulary-sharded forward: 4 slices of W + merge
+    spec = workloads.spec_for(CONFIG_ID)
+    wl = workloads.build(spec, "cuda")
+    h, w, y = wl.hidden, wl.w_vocab, wl.targets
+    Nt, d, V, P = wl.N, spec.d, spec.V, 4
+    bounds = [V * p // P for p in range(P + 1)]
+    states = torch.empty((P, Nt, 4), dtype=torch.float32, device="cuda")
+    ws = torch.empty(mc.forward_workspace_size(Nt, d, max(b - a for a, b in zip(bounds[:-1], bounds[1:]))),
+                     dtype=torch.uint8, device="cuda")
+    slices = [w[a:b] for a, b in zip(bounds[:-1], bounds[1:])]
+
+    def shard_calls():
+        for p in range(P):
+            mc.token_logprob_state(h, slices[p], y, bounds[p], 1.0, state=states[p], workspace=ws)
+
+    merged = mc.merge_logprob_states(states)
+    ms_s = _time_calls(shard_calls, args.launches)
+    ms_m = _time_calls(lambda: mc.merge_logprob_states(states, out=merged), args.launches)
+    flop = 2.0 * Nt * d * V
+    res["sharded_forward"] = {"tokens": Nt, "slices": P, "ms_slices": ms_s, "tflops": flop / (ms_s / 1e3) / 1e12,
+                              "frac_of_sustained": flop / (ms_s / 1e3) / 1e12 / peaks["bf16_sustained"],
+                              "merge_ms": ms_m, "merge_bytes_per_token": 16 * P + 12,
+                              "merge_gbs": (16 * P + 12) * Nt / (ms_m / 1e3) / 1e9}
+    del wl, h, w, y, states, ws, slices, merged
+    torch.cuda.empty_cache()
+
+    # PrimeEcho reward + group advantage
+    res["advantage"] = {}
+    for T in (512, 1 << 24):
+        K, G = 4, 8
+        gg = torch.Generator(device="cuda").manual_seed(1)
+        scores = torch.rand((T, K), generator=gg, device="cuda") * 2 - 0.5
+        success = (torch.rand((T, K), generator=gg, device="cuda") < 0.3).to(torch.uint8)
+        n_turns = torch.randint(1, K + 1, (T,), generator=gg, device="cuda", dtype=torch.int32)
+        ms_a = _time_calls(lambda: mc.prime_echo_advantages(scores, success, n_turns, G, 0.75, 0.5, 0.2),
+                           args.launches)
+        bpt = 5 * K + 4 + 8
+        res["advantage"][str(T)] = {"trajectories": T, "turns": K, "group": G, "us": ms_a * 1e3,
+                                    "bytes_per_trajectory": bpt, "achieved_gbs": bpt * T / (ms_a / 1e3) / 1e9}
+    print(json.dumps(res), flush=True)
+
+
 def run_case(args):
     """One call of the path, `--launches` times, for ncu captures (no timing printed
     beyond a one-line summary): --case fwd|bwd|filter|loss on the first `--rows`
@@ -559,6 +653,8 @@ def run_case(args):
 
     if args.case == "stream":
         return run_stream(args)
+    if args.case == "next":
+        return run_next(args)
     torch.cuda.set_device(0)
     if not os.path.exists(mc.lib_path()):
         mcbuild.build()
@@ -643,7 +739,7 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=384)
     ap.add_argument("--ref-rows", type=int, default=64)
-    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream"], default="step",
+    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream", "next"], default="step",
                     help="profiling aid: run one call of the path --launches times")
     ap.add_argument("--rows", type=int, default=0, help="--case: tokens to use (0 = the whole batch)")
     ap.add_argument("--launches", type=int, default=2)

@@ -6,9 +6,12 @@
 //         + beta1 1[success_{i,1}] + beta2 1[!success_{i,1} && success_{i,2}]
 //   A_i = (R_i - mean_G R) / (std_G R + eps),  std with divisor G - 1
 //
-// One thread per group of G consecutive trajectories (a few hundred groups per
-// batch): it forms the G rewards, then the mean and the standard deviation in
-// two passes. Latency-bound by design.
+// Group sizes dividing 32 (the paper's G = 8 among them): one thread per
+// trajectory, a group's G trajectories on G consecutive lanes of a warp (a
+// group never straddles two warps), its mean and standard deviation formed by
+// xor-shuffle butterflies inside those lanes; a warp reads 32 consecutive
+// trajectory rows. Other group sizes: one thread per group forms the G
+// rewards, then the mean and the standard deviation in two passes.
 #include "mc_internal.h"
 
 namespace mc {
@@ -54,10 +57,47 @@ __global__ void __launch_bounds__(kAdvThreads) group_advantage_kernel(AdvArgs p)
   }
 }
 
+template <int G>
+__global__ void __launch_bounds__(kAdvThreads) group_advantage_lanes_kernel(AdvArgs p) {
+  static_assert(32 % G == 0, "a group must fit the lanes of one warp");
+  const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool live = i < p.n_groups * G;  // whole groups: the tail's dead lanes form dead groups
+  const float r = live ? trajectory_reward(p, i) : 0.f;
+  float sum = r;
+#pragma unroll
+  for (int off = G / 2; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+  const float mean = sum / static_cast<float>(G);
+  const float dv = r - mean;
+  float ss = dv * dv;
+#pragma unroll
+  for (int off = G / 2; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  if (!live) return;
+  const float sd = G > 1 ? sqrtf(ss / static_cast<float>(G - 1)) : 0.f;
+  if (p.reward) p.reward[i] = r;
+  p.advantage[i] = (G > 1 && sd + p.eps > 0.f) ? dv * (1.f / (sd + p.eps)) : 0.f;
+}
+
+template <int G>
+cudaError_t launch_lanes(const AdvArgs& a, cudaStream_t stream) {
+  const long long T = a.n_groups * G;
+  const long long blocks = (T + kAdvThreads - 1) / kAdvThreads;
+  group_advantage_lanes_kernel<G><<<static_cast<unsigned>(blocks), kAdvThreads, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_group_advantage(const AdvArgs& a, cudaStream_t stream) {
   if (a.n_groups <= 0) return cudaSuccess;
+  switch (a.G) {
+    case 1: return launch_lanes<1>(a, stream);
+    case 2: return launch_lanes<2>(a, stream);
+    case 4: return launch_lanes<4>(a, stream);
+    case 8: return launch_lanes<8>(a, stream);
+    case 16: return launch_lanes<16>(a, stream);
+    case 32: return launch_lanes<32>(a, stream);
+    default: break;
+  }
   const long long blocks = (a.n_groups + kAdvThreads - 1) / kAdvThreads;
   group_advantage_kernel<<<static_cast<unsigned>(blocks), kAdvThreads, 0, stream>>>(a);
   return cudaGetLastError();

@@ -1,7 +1,8 @@
 """GPU PrimeEcho reward / group advantage (mc_prime_echo_advantages) vs the
 fp64 oracle: the paper's batch shape (64 prompts x G = 8, up to K = 3 turns),
-the alpha = 1 / alpha = 0 cases, single-turn GRPO (Eq. 3) and degenerate
-groups. Tolerance: 1e-5 absolute on rewards, 1e-4 absolute on advantages
+the alpha = 1 / alpha = 0 cases, single-turn GRPO (Eq. 3), degenerate
+groups, group sizes reduced across warp lanes (dividing 32, with a partial
+last warp) and others (one thread per group). Tolerance: 1e-5 absolute on rewards, 1e-4 absolute on advantages
 (fp32 two-pass mean / std of O(1) values)."""
 
 import numpy as np
@@ -51,3 +52,8 @@ def test_degenerate_groups():
     out = check(scores, success, torch.full((16,), 2, dtype=torch.int32), 8, 0.75, 0.5, 0.2, 1e-6)
     assert not out["advantage"].any()
     check(*make(5, 3, 2), 1, 0.75, 0.5, 0.2, 1e-6)  # groups of one: advantage 0
+
+
+@pytest.mark.parametrize("T,G", [(40, 8), (96, 32), (48, 16), (34, 2), (60, 6), (36, 12), (1 << 16, 8)])
+def test_group_sizes_and_batch_tails(T, G):
+    check(*make(T, 4, 3), G, 0.75, 0.5, 0.2, 1e-6)
