@@ -57,12 +57,29 @@ __global__ void __launch_bounds__(kAdvThreads) group_advantage_kernel(AdvArgs p)
   }
 }
 
+// K = 4 turns with aligned arrays: one 16-byte load of the row's scores and
+// one 4-byte load of its success flags.
+__device__ __forceinline__ float trajectory_reward4(const AdvArgs& p, long long i) {
+  int k = p.n_turns[i];
+  k = k < 1 ? 1 : (k > 4 ? 4 : k);
+  const float4 s = reinterpret_cast<const float4*>(p.scores)[i];
+  const uchar4 ok = reinterpret_cast<const uchar4*>(p.success)[i];
+  float best = s.x;
+  if (k >= 2) best = fmaxf(best, s.y);
+  if (k >= 3) best = fmaxf(best, s.z);
+  if (k >= 4) best = fmaxf(best, s.w);
+  const bool first_ok = ok.x != 0;
+  const bool second_ok = k >= 2 && ok.y != 0;
+  const float bonus = (first_ok ? p.beta1 : 0.f) + ((!first_ok && second_ok) ? p.beta2 : 0.f);
+  return p.alpha * s.x + (1.f - p.alpha) * best + bonus;
+}
+
 template <int G>
 __global__ void __launch_bounds__(kAdvThreads) group_advantage_lanes_kernel(AdvArgs p) {
   static_assert(32 % G == 0, "a group must fit the lanes of one warp");
   const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
   const bool live = i < p.n_groups * G;  // whole groups: the tail's dead lanes form dead groups
-  const float r = live ? trajectory_reward(p, i) : 0.f;
+  const float r = !live ? 0.f : (p.vec4 ? trajectory_reward4(p, i) : trajectory_reward(p, i));
   float sum = r;
 #pragma unroll
   for (int off = G / 2; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);

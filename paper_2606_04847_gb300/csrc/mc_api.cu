@@ -625,6 +625,7 @@ mc_status mc_prime_echo_advantages(const float* scores, const uint8_t* success, 
   a.eps = eps;
   a.reward = reward;
   a.advantage = advantage;
+  a.vec4 = (K == 4 && aligned(scores, 16) && aligned(success, 4)) ? 1 : 0;
   cudaError_t e = mc::launch_group_advantage(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "advantage launch");
   return MC_OK;

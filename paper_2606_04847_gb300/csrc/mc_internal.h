@@ -172,6 +172,7 @@ struct AdvArgs {
   float alpha, beta1, beta2, eps;
   float* reward;           // [T] or null
   float* advantage;        // [T]
+  int vec4;                // K == 4, scores 16-byte and success 4-byte aligned: vector row loads
 };
 cudaError_t launch_group_advantage(const AdvArgs& a, cudaStream_t stream);
 

@@ -55,5 +55,16 @@ def test_degenerate_groups():
 
 
 @pytest.mark.parametrize("T,G", [(40, 8), (96, 32), (48, 16), (34, 2), (60, 6), (36, 12), (1 << 16, 8)])
-def test_group_sizes_and_batch_tails(T, G):
-    check(*make(T, 4, 3), G, 0.75, 0.5, 0.2, 1e-6)
+@pytest.mark.parametrize("K", [4, 3])  # 4 turns: vector row loads; 3: per-turn loads
+def test_group_sizes_and_batch_tails(T, G, K):
+    check(*make(T, K, 3), G, 0.75, 0.5, 0.2, 1e-6)
+
+
+def test_four_turns_unaligned_rows_take_the_scalar_path():
+    scores, success, n_turns = make(65, 4, 4)
+    sc = torch.empty(65 * 4 + 1).cuda()[1:].view(65, 4)  # rows 4 bytes off a 16-byte boundary
+    sc.copy_(scores.cuda())
+    out = mc.prime_echo_advantages(sc, success.cuda(), n_turns.cuda(), 5, 0.75, 0.5, 0.2, 1e-6)
+    ref = mc.prime_echo_advantages(scores.cuda(), success.cuda(), n_turns.cuda(), 5, 0.75, 0.5, 0.2, 1e-6)
+    torch.cuda.synchronize()
+    torch.testing.assert_close(out["advantage"], ref["advantage"], rtol=0, atol=1e-6)
