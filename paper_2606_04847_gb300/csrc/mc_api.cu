@@ -17,13 +17,12 @@
 
 #include "mc.h"
 #include "mc_internal.h"
+#include "mc_schedule.h"
 
 namespace {
 
-constexpr int kBM = 128;       // rows one CTA owns in a tile (TMA box height for A)
-constexpr int kBN = 256;       // vocabulary / output columns per tile
-constexpr int kRowPad = 256;   // row padding of workspaces: one row block of either engine
-constexpr int kMaxSplits = 16;
+using namespace mc::sched;
+
 constexpr size_t kStatusBytes = 256;
 constexpr int kMaxDevices = 64;
 
@@ -35,7 +34,6 @@ mc_status cuda_fail(cudaError_t e, const char* what) {
 }
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // ---- cached device attributes (the only state the library keeps)
@@ -77,32 +75,6 @@ uint64_t wait_timeout_ns() {
   }();
   return t;
 }
-
-// The one-CTA engine unless MC_ENGINE=pair selects the CTA-pair engine
-// (tcgen05 cta_group::2). Both give the same results; under the GB300's power
-// cap the one-CTA engine sustains a ~10 % higher SM clock and is ~4 % faster
-// on the 9B-class forward, so it is the default.
-bool use_pair_engine() {
-  static const bool pair = [] {
-    const char* s = std::getenv("MC_ENGINE");
-    return s != nullptr && std::strcmp(s, "pair") == 0;
-  }();
-  return pair;
-}
-
-// Projection launches (forward, dZ) of the one-CTA engine with at least this
-// many rows use 256-row tiles (TileCfg<2>: a third less operand traffic per
-// FLOP, 8 epilogue warps); fewer rows keep 128-row tiles so that small
-// launches still spread over the SMs.
-constexpr long long kWideMinRows = 4096;
-bool wide_rows(long long rows) { return !use_pair_engine() && rows >= kWideMinRows; }
-
-// Rows per scheduled row block of a projection launch over `rows` rows, TMA
-// box height of K-major B, and how many units run at once, for the selected
-// engine.
-int row_block(long long rows) { return (use_pair_engine() || wide_rows(rows)) ? 256 : kBM; }
-int b_box_rows() { return use_pair_engine() ? 128 : kBN; }
-int concurrent_units(int sms) { return use_pair_engine() ? sms / 2 : sms; }
 
 // ---- TMA descriptors
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -152,37 +124,6 @@ mc_status make_tmap_box(CUtensorMap* m, const void* base, uint64_t inner, uint64
 mc_status make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_elems,
                     uint32_t box_outer) {
   return make_tmap_box(m, base, inner, outer, stride_elems, 64, box_outer, CU_TENSOR_MAP_SWIZZLE_128B);
-}
-
-// Vocabulary tile ranges per row block. A wave of `conc` concurrent units
-// streams W once and keeps its conc / s row blocks of hidden rows in L2, so
-// s is at least the count that holds those rows under kWaveRowBytes. Among
-// the counts allowed, the one with the shortest critical path in tiles,
-// waves(s) x ceil(n_tiles / s); counts within 0.5 % of the best resolve to
-// the fewest splits (fewest W streams).
-constexpr double kWaveRowBytes = 40.0 * (1 << 20);
-
-int choose_splits(long long m_blocks, int n_tiles, int conc, int rb, int d) {
-  long long lo = static_cast<long long>(std::ceil(double(conc) * rb * d * 2.0 / kWaveRowBytes));
-  if (lo < 1) lo = 1;
-  long long hi = kMaxSplits;
-  if (hi > n_tiles) hi = n_tiles;
-  if (lo > hi) lo = hi;
-  double best_path = 0.0;
-  for (long long s = lo; s <= hi; ++s) {
-    const double path = double(ceil_div(m_blocks * s, conc)) * double(ceil_div(n_tiles, s));
-    if (s == lo || path < best_path) best_path = path;
-  }
-  for (long long s = lo; s <= hi; ++s) {
-    const double path = double(ceil_div(m_blocks * s, conc)) * double(ceil_div(n_tiles, s));
-    if (path <= best_path * 1.005) return static_cast<int>(s);
-  }
-  return static_cast<int>(hi);
-}
-
-int max_splits(int V) {
-  const int n_tiles = static_cast<int>(ceil_div(V, kBN));
-  return n_tiles < kMaxSplits ? n_tiles : kMaxSplits;
 }
 
 bool valid_common(int64_t N, int32_t d, int32_t V, float inv_temperature) {
