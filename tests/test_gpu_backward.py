@@ -101,6 +101,12 @@ def test_wide_tile_dz_producer():
     check(*setup(4500, 128, 1500, seed=14), inv_temp=1.0 / 0.9)
 
 
+def test_wide_tile_dz_tiny_vocabulary_single_k_block():
+    """dZ on 256-row tiles with V = 17 (a 17-column store box, clipped by the
+    tensor map) and d = 64 (one k-block per tile)."""
+    check(*setup(4500, 64, 17, seed=17))
+
+
 def test_wide_tile_dz_27b_hidden_size():
     """256-row dZ tiles at d = 5120 (80 k-blocks per tile), 4500 rows (a
     ragged last 32-row store box), V = 700 (a 28-column last store box)."""

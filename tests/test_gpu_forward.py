@@ -57,6 +57,13 @@ def test_wide_tiles_ragged(inv_temp):
     run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
 
 
+def test_wide_tiles_tiny_vocabulary_single_k_block():
+    """256-row tiles with V = 17 (less than one 32-column chunk) and d = 64
+    (one k-block per tile)."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=4500, len_hi=4500, d=64, V=17)
+    run_and_compare(workloads.build(spec, "cpu"))
+
+
 @pytest.mark.parametrize("N,V", [(127, 1), (128, 31), (129, 33), (5, 257)])
 def test_tiny_vocabularies_and_block_edges(N, V):
     """V = 1 (logp = 0, entropy = 0), V inside the first 32-column chunk, N on
