@@ -113,6 +113,28 @@ def _need(t: torch.Tensor, name: str, dtype, ndim: int):
         raise ValueError(f"{name} must be a contiguous {ndim}-d tensor")
 
 
+def _shaped(t: Optional[torch.Tensor], name: str, dtype, shape, device) -> Optional[torch.Tensor]:
+    """Checks a caller-supplied tensor (None passes): dtype, device, contiguity
+    and exact shape, so that no kernel writes or reads past its end."""
+    if t is None:
+        return None
+    _need(t, name, dtype, len(shape))
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if t.device != device:
+        raise ValueError(f"{name} must be on {device}, got {t.device}")
+    return t
+
+
+def _ws(t: torch.Tensor, device) -> torch.Tensor:
+    """A caller-supplied workspace: uint8, 1-d, contiguous, on `device` (its
+    size is checked by the library against the call's requirement)."""
+    _need(t, "workspace", torch.uint8, 1)
+    if t.device != device:
+        raise ValueError(f"workspace must be on {device}, got {t.device}")
+    return t
+
+
 def version() -> tuple:
     v = lib().mc_version()
     return (v >> 16, v & 0xFFFF)
@@ -139,11 +161,17 @@ def token_logprobs(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: torch.T
     if w_vocab.shape[1] != d or targets.shape[0] != N:
         raise ValueError("shape mismatch")
     dev = hidden.device
+    _shaped(w_vocab, "w_vocab", torch.bfloat16, (V, d), dev)
+    _shaped(targets, "targets", torch.int32, (N,), dev)
     if out is None:
         out = {k: torch.empty(N, dtype=torch.float32, device=dev) for k in ("logp", "entropy", "lse")}
+    _shaped(out["logp"], "out['logp']", torch.float32, (N,), dev)
+    for k in ("entropy", "lse"):
+        _shaped(out.get(k), f"out['{k}']", torch.float32, (N,), dev)
     need = forward_workspace_size(N, d, V)
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    _ws(workspace, dev)
     st = lib().mc_token_logprobs(_ptr(hidden), _ptr(w_vocab), _ptr(targets), N, d, V, float(inv_temperature),
                                  _ptr(out["logp"]), _ptr(out.get("entropy")), _ptr(out.get("lse")),
                                  _ptr(workspace), workspace.numel(), _ptr(dev_status), _stream(stream))
@@ -161,10 +189,15 @@ def token_logprob_state(hidden: torch.Tensor, w_shard: torch.Tensor, targets: to
     _need(targets, "targets", torch.int32, 1)
     N, d = hidden.shape
     Vs = w_shard.shape[0]
+    dev = hidden.device
+    _shaped(w_shard, "w_shard", torch.bfloat16, (Vs, d), dev)
+    _shaped(targets, "targets", torch.int32, (N,), dev)
     if state is None:
-        state = torch.empty((N, 4), dtype=torch.float32, device=hidden.device)
+        state = torch.empty((N, 4), dtype=torch.float32, device=dev)
+    _shaped(state, "state", torch.float32, (N, 4), dev)
     if workspace is None:
-        workspace = torch.empty(max(forward_workspace_size(N, d, Vs), 256), dtype=torch.uint8, device=hidden.device)
+        workspace = torch.empty(max(forward_workspace_size(N, d, Vs), 256), dtype=torch.uint8, device=dev)
+    _ws(workspace, dev)
     st = lib().mc_token_logprob_state(_ptr(hidden), _ptr(w_shard), _ptr(targets), N, d, Vs, int(v_begin),
                                       float(inv_temperature), _ptr(state), _ptr(workspace), workspace.numel(),
                                       _ptr(dev_status), _stream(stream))
@@ -181,6 +214,9 @@ def merge_logprob_states(states: torch.Tensor, *, out: Optional[dict] = None,
         raise ValueError("states must be [P, N, 4]")
     if out is None:
         out = {k: torch.empty(N, dtype=torch.float32, device=states.device) for k in ("logp", "entropy", "lse")}
+    _shaped(out["logp"], "out['logp']", torch.float32, (N,), states.device)
+    for k in ("entropy", "lse"):
+        _shaped(out.get(k), f"out['{k}']", torch.float32, (N,), states.device)
     st = lib().mc_merge_logprob_states(_ptr(states), P, N, _ptr(out["logp"]), _ptr(out.get("entropy")),
                                        _ptr(out.get("lse")), _ptr(dev_status), _stream(stream))
     _check("mc_merge_logprob_states", st)
@@ -202,6 +238,12 @@ def token_logprobs_noalloc(hidden: torch.Tensor, w_vocab: torch.Tensor, targets:
     _need(targets, "targets", torch.int32, 1)
     N, d = hidden.shape
     V = w_vocab.shape[0]
+    dev = hidden.device
+    _shaped(w_vocab, "w_vocab", torch.bfloat16, (V, d), dev)
+    _shaped(targets, "targets", torch.int32, (N,), dev)
+    _shaped(out["logp"], "out['logp']", torch.float32, (N,), dev)
+    for k in ("entropy", "lse"):
+        _shaped(out.get(k), f"out['{k}']", torch.float32, (N,), dev)
     st = lib().mc_token_logprobs_noalloc(_ptr(hidden), _ptr(w_vocab), _ptr(targets), N, d, V,
                                          float(inv_temperature), _ptr(out["logp"]), _ptr(out.get("entropy")),
                                          _ptr(out.get("lse")), _ptr(dev_status), _stream(stream))
@@ -228,13 +270,23 @@ def token_logprobs_bwd(hidden: torch.Tensor, w_vocab: torch.Tensor, targets: tor
     N, d = hidden.shape
     V = w_vocab.shape[0]
     dev = hidden.device
+    _shaped(w_vocab, "w_vocab", torch.bfloat16, (V, d), dev)
+    _shaped(targets, "targets", torch.int32, (N,), dev)
+    _shaped(lse, "lse", torch.float32, (N,), dev)
+    _shaped(entropy, "entropy", torch.float32, (N,), dev)
+    _shaped(grad_logp, "grad_logp", torch.float32, (N,), dev)
+    _shaped(grad_entropy, "grad_entropy", torch.float32, (N,), dev)
+    _shaped(row_keep, "row_keep", torch.uint8, (N,), dev)
     if grad_hidden is None:
         grad_hidden = torch.empty((N, d), dtype=torch.bfloat16, device=dev)
     if grad_w is None:
         grad_w = torch.empty((V, d), dtype=torch.float32, device=dev)
+    _shaped(grad_hidden, "grad_hidden", torch.bfloat16, (N, d), dev)
+    _shaped(grad_w, "grad_w", torch.float32, (V, d), dev)
     if workspace is None:
         need = backward_workspace_size(N, d, V, rows_per_chunk)
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    _ws(workspace, dev)
     st = lib().mc_token_logprobs_bwd(_ptr(hidden), _ptr(w_vocab), _ptr(targets), _ptr(lse), _ptr(entropy),
                                      _ptr(grad_logp), _ptr(grad_entropy), _ptr(row_keep), N, d, V,
                                      float(inv_temperature),
@@ -267,6 +319,15 @@ def seq_ratio_filter(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
         if token_outputs:
             out["token_ratio"] = torch.empty(N, dtype=torch.float32, device=dev)
             out["token_keep"] = torch.empty(N, dtype=torch.uint8, device=dev)
+    _shaped(logp_behaviour, "logp_behaviour", torch.float32, (N,), dev)
+    _shaped(loss_mask, "loss_mask", torch.uint8, (N,), dev)
+    _shaped(cu_seqlens, "cu_seqlens", torch.int64, (B + 1,), dev)
+    for k, dt, n in (("signed_mean", torch.float32, B), ("abs_mean", torch.float32, B), ("n_tokens", torch.int32, B),
+                     ("keep", torch.uint8, B), ("keep_vanilla", torch.uint8, B), ("token_ratio", torch.float32, N),
+                     ("token_keep", torch.uint8, N)):
+        if k in ("signed_mean", "abs_mean", "n_tokens", "keep") and out.get(k) is None:
+            raise ValueError(f"out['{k}'] is required")
+        _shaped(out.get(k), f"out['{k}']", dt, (n,), dev)
     st = lib().mc_seq_ratio_filter(_ptr(logp_policy), _ptr(logp_behaviour), _ptr(loss_mask), _ptr(cu_seqlens),
                                    B, N, float(delta), float(delta_vanilla), _ptr(out["signed_mean"]),
                                    _ptr(out["abs_mean"]), _ptr(out["n_tokens"]), _ptr(out["keep"]),
@@ -301,8 +362,21 @@ def grpo_masked_loss(logp_policy: torch.Tensor, logp_behaviour: torch.Tensor, lo
                "seq_loss": torch.empty(B, dtype=torch.float32, device=dev),
                "n_clipped": torch.empty(1, dtype=torch.int32, device=dev),
                "kl": torch.empty(1, dtype=torch.float32, device=dev)}
+    _shaped(logp_behaviour, "logp_behaviour", torch.float32, (N,), dev)
+    _shaped(logp_ref, "logp_ref", torch.float32, (N,), dev)
+    _shaped(loss_mask, "loss_mask", torch.uint8, (N,), dev)
+    _shaped(cu_seqlens, "cu_seqlens", torch.int64, (B + 1,), dev)
+    _shaped(advantages, "advantages", torch.float32, (B,), dev)
+    _shaped(keep, "keep", torch.uint8, (B,), dev)
+    _shaped(n_tokens, "n_tokens", torch.int32, (B,), dev)
+    for k, dt, n in (("loss", torch.float32, 1), ("grad_logp", torch.float32, N), ("seq_loss", torch.float32, B),
+                     ("n_clipped", torch.int32, 1), ("kl", torch.float32, 1)):
+        if k in ("loss", "grad_logp") and out.get(k) is None:
+            raise ValueError(f"out['{k}'] is required")
+        _shaped(out.get(k), f"out['{k}']", dt, (n,), dev)
     if workspace is None:
         workspace = torch.empty(lib().mc_grpo_masked_loss_workspace_size(B), dtype=torch.uint8, device=dev)
+    _ws(workspace, dev)
     st = lib().mc_grpo_masked_loss(_ptr(logp_policy), _ptr(logp_behaviour), _ptr(loss_mask), _ptr(cu_seqlens),
                                    _ptr(advantages), _ptr(keep), _ptr(n_tokens), B, N, float(eps_low),
                                    float(eps_high), _ptr(logp_ref), float(beta), _ptr(out["loss"]),
@@ -320,8 +394,8 @@ def prime_echo_advantages(scores: torch.Tensor, success: torch.Tensor, n_turns: 
     _need(success, "success", torch.uint8, 2)
     _need(n_turns, "n_turns", torch.int32, 1)
     T, K = scores.shape
-    if success.shape != (T, K) or n_turns.shape[0] != T:
-        raise ValueError("shape mismatch")
+    _shaped(success, "success", torch.uint8, (T, K), scores.device)
+    _shaped(n_turns, "n_turns", torch.int32, (T,), scores.device)
     out = {"reward": torch.empty(T, dtype=torch.float32, device=scores.device),
            "advantage": torch.empty(T, dtype=torch.float32, device=scores.device)}
     st = lib().mc_prime_echo_advantages(_ptr(scores), _ptr(success), _ptr(n_turns), T, K, int(group_size),

@@ -144,3 +144,28 @@ def test_bounded_wait_selftest_keeps_context_usable():
     torch.cuda.synchronize()
     assert int(st.item()) & mc.MC_DEV_TIMEOUT
     test_config1_tiny_full_size()  # the context is still healthy
+
+
+def test_binding_rejects_mis_shaped_outputs_and_workspaces():
+    """Caller-supplied outputs and workspaces are checked before any launch: a
+    wrong shape, dtype or layout raises instead of letting a kernel write past
+    a buffer."""
+    wl = workloads.build(workloads.spec_for(1, n_seqs=1, len_lo=64, len_hi=64, d=64, V=256), "cpu")
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    with pytest.raises(ValueError):
+        mc.token_logprobs(h, w, y, out={"logp": torch.empty(63, device="cuda")})
+    with pytest.raises(TypeError):
+        mc.token_logprobs(h, w, y, out={"logp": torch.empty(64, device="cuda", dtype=torch.float64)})
+    with pytest.raises(TypeError):
+        mc.token_logprobs(h, w, y, workspace=torch.empty(1 << 20, device="cuda", dtype=torch.float32))
+    with pytest.raises(ValueError):
+        mc.token_logprobs(h, w.t().contiguous().t(), y)  # a strided view of W
+    fw = mc.token_logprobs(h, w, y)
+    g = torch.randn(64, device="cuda")
+    with pytest.raises(ValueError):
+        mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g, grad_w=torch.empty(256, 32, device="cuda"))
+    with pytest.raises(ValueError):
+        mc.token_logprobs_bwd(h, w, y, fw["lse"][:10], fw["entropy"], g)
+    cu = torch.tensor([0, 64], dtype=torch.int64, device="cuda")
+    with pytest.raises(ValueError):
+        mc.seq_ratio_filter(fw["logp"], fw["logp"][:32], None, cu, 0.1)
