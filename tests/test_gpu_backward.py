@@ -147,6 +147,22 @@ def test_peaked_softmax():
     check(*setup(256, 256, 2048, seed=6, w_scale=8.0))
 
 
+def test_extreme_logits():
+    """W x 64: the softmax is nearly one-hot, dZ nearly g (1[v = y] - 1[v = argmax])."""
+    check(*setup(300, 128, 1500, seed=18, w_scale=64.0))
+
+
+@pytest.mark.parametrize("N", [450, 4500])  # 128-row and 256-row dZ tiles
+def test_deterministic_bitwise(N):
+    """No atomics, fixed reduction orders: two calls give identical bits."""
+    wl, g, ge = setup(N, 128, 1000, seed=19)
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    fw = mc.token_logprobs(h, w, y)
+    a = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda())
+    b = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda())
+    assert torch.equal(a["grad_hidden"], b["grad_hidden"]) and torch.equal(a["grad_w"], b["grad_w"])
+
+
 def test_row_keep_gate_equals_zeroed_upstream():
     """row_keep = 0 on a dropped sequence gives the same gradients as zeroing
     its upstream gradient (the M_i factor of Eq. 17)."""

@@ -90,6 +90,16 @@ def test_peaked_softmax_low_entropy():
     assert ref["entropy"].min() < 0.5
 
 
+@pytest.mark.parametrize("N", [300, 4500])  # 128-row and 256-row tiles
+def test_extreme_logits(N):
+    """W x 64: logits spread over hundreds of units, so nearly every row is
+    one-hot-dominant and the running maximum jumps between tiles; exp2 of
+    very negative arguments flushes to 0."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=128, V=2000, w_scale=64.0)
+    out, ref = run_and_compare(workloads.build(spec, "cpu"))
+    assert ref["entropy"].min() < 1e-3
+
+
 def test_uniform_logits():
     """W = 0: every logit equal; logp = -log V and entropy = log V."""
     N, d, V = 130, 64, 777
