@@ -43,7 +43,7 @@ typedef struct CUstream_st* mc_stream_t;
 typedef enum {
   MC_OK = 0,
   MC_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, size out of range */
-  MC_ERR_UNSUPPORTED = 2,   /* valid request this build does not run (e.g. d % 64 != 0, no sm_103 GPU) */
+  MC_ERR_UNSUPPORTED = 2,   /* a valid request the library does not run (e.g. no sm_103 GPU) */
   MC_ERR_CUDA = 3,          /* a CUDA runtime or driver call failed; see mc_last_cuda_error() */
   MC_ERR_TIMEOUT = 4,       /* reported through dev_status: see MC_DEV_TIMEOUT */
   MC_ERR_WORKSPACE = 5,     /* workspace pointer null/misaligned or smaller than the query */
