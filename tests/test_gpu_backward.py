@@ -178,3 +178,32 @@ def test_row_keep_gate_equals_zeroed_upstream():
     assert torch.equal(a["grad_w"], b["grad_w"])
     ref = oracle.token_logprobs_bwd(wl.hidden, wl.w_vocab, wl.targets, g0, ge0)
     assert rel_fro(np_(a["grad_w"]), ref["grad_w"]) <= TOL_GRAD
+
+
+@pytest.mark.parametrize("N", [300, 16500])  # grad_w on 128-row and on 256-row tiles
+def test_every_row_dropped(N):
+    """row_keep all 0: no row has a gradient, so the device-side K of grad_w is
+    0: grad_hidden and grad_w are zero, or grad_w keeps its value when
+    accumulating."""
+    wl, g, ge = setup(N, 64, 300, seed=20)
+    h, w, y = wl.hidden.cuda(), wl.w_vocab.cuda(), wl.targets.cuda()
+    fw = mc.token_logprobs(h, w, y)
+    keep = torch.zeros(N, dtype=torch.uint8, device="cuda")
+    out = mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda(), row_keep=keep)
+    torch.cuda.synchronize()
+    assert not out["grad_hidden"].any() and not out["grad_w"].any()
+    base = torch.randn(300, 64, device="cuda")
+    gw = base.clone()
+    mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], g.cuda(), ge.cuda(), row_keep=keep, grad_w=gw,
+                          accumulate=True)
+    torch.cuda.synchronize()
+    assert torch.equal(gw, base)
+
+
+def test_zero_rows():
+    wl, g, _ = setup(8, 64, 300, seed=21)
+    h, w, y = wl.hidden.cuda()[:0], wl.w_vocab.cuda(), wl.targets.cuda()[:0]
+    z = torch.empty(0, device="cuda")
+    out = mc.token_logprobs_bwd(h, w, y, z, None, z)
+    torch.cuda.synchronize()
+    assert out["grad_hidden"].shape == (0, 64) and not out["grad_w"].any()
