@@ -1,15 +1,16 @@
 // mc_filter.cu — per-sequence importance-ratio statistics and the MirrorPop
 // keep-mask (§4.5.2, Eq. 18-21), plus per-token ratios (Eq. 4).
 //
-// Persistent CTAs (8 per SM) stride over the sequences, one sequence at a
-// time per CTA. Each thread walks its share of the sequence's packed tokens
+// Persistent CTAs (16 per SM, 128 threads each) stride over the sequences, one
+// sequence at a time per CTA. Each thread walks its share of the sequence's packed tokens
 // with 16-byte loads (4 tokens of logp_policy / logp_behaviour, 4 mask bytes;
 // two vectors in flight), accumulates sum(log rho), sum(|log rho|) and the
 // count over loss-masked tokens, and writes rho = exp(log rho) on the way
 // (streaming stores). Warp shuffles then
 // a shared-memory step reduce the three sums in a fixed order (deterministic
 // for a given launch shape). Thread 0 forms the statistics and the masks; a
-// second sweep writes token_keep once keep_i is known. The kernel is HBM-
+// second sweep writes token_keep once keep_i is known, 16 tokens per 16-byte
+// load of the mask and store. The kernel is HBM-
 // bound: 4 + 4 + 1 bytes read and up to 4 + 1 bytes written per token.
 #include "mc_internal.h"
 #include "mc_ptx.cuh"
@@ -42,6 +43,16 @@ __device__ __forceinline__ void add_vec(Acc& acc, const float4& lp, const float4
   if (mk.y) { acc.s += d1; acc.a += fabsf(d1); acc.n += 1; }
   if (mk.z) { acc.s += d2; acc.a += fabsf(d2); acc.n += 1; }
   if (mk.w) { acc.s += d3; acc.a += fabsf(d3); acc.n += 1; }
+}
+
+// 0x01 in every byte of w that is nonzero, 0x00 elsewhere: the low seven bits
+// of a byte plus 0x7F reach bit 7 exactly when they are not all zero (no carry
+// leaves the byte), and OR-ing the byte itself covers its own bit 7.
+__device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
+  return ((((w & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | w) & 0x80808080u) >> 7;
+}
+__device__ __forceinline__ uint4 nonzero_bytes(uint4 v) {
+  return make_uint4(nonzero_bytes(v.x), nonzero_bytes(v.y), nonzero_bytes(v.z), nonzero_bytes(v.w));
 }
 
 // Persistent over sequences (CTA c handles sequences c, c + gridDim.x, ...).
@@ -123,7 +134,23 @@ __global__ void __launch_bounds__(kFilterThreads) seq_filter_kernel(FilterArgs p
     __syncthreads();
     if (p.token_keep != nullptr) {
       const uint8_t k = static_cast<uint8_t>(keep_s);
-      for (long long t = b + threadIdx.x; t < e; t += blockDim.x)
+      // token_keep = keep_i & (mask != 0): scalar up to a 16-token boundary,
+      // then 16 tokens per 16-byte load / store, then the tail (all scalar
+      // when the bases are not 16-byte aligned).
+      long long hb = p.keep_vec_ok ? ((b + 15) & ~15LL) : e;
+      if (hb > e) hb = e;
+      const long long vend = hb + ((e - hb) & ~15LL);
+      for (long long t = b + threadIdx.x; t < hb; t += blockDim.x)
+        p.token_keep[t] = static_cast<uint8_t>(k & (p.loss_mask ? (p.loss_mask[t] != 0) : 1));
+      const uint4* m16 = reinterpret_cast<const uint4*>(p.loss_mask);
+      uint4* k16 = reinterpret_cast<uint4*>(p.token_keep);
+      for (long long q = (hb >> 4) + threadIdx.x; q < (vend >> 4); q += blockDim.x) {
+        uint4 o = make_uint4(0u, 0u, 0u, 0u);
+        if (k) o = p.loss_mask ? nonzero_bytes(m16[q]) : make_uint4(0x01010101u, 0x01010101u, 0x01010101u,
+                                                                    0x01010101u);
+        k16[q] = o;
+      }
+      for (long long t = vend + threadIdx.x; t < e; t += blockDim.x)
         p.token_keep[t] = static_cast<uint8_t>(k & (p.loss_mask ? (p.loss_mask[t] != 0) : 1));
     }
     __syncthreads();  // warp_acc / keep_s are reused by the next sequence

@@ -133,6 +133,7 @@ struct FilterArgs {
   float* token_ratio;
   uint8_t* token_keep;
   int vec_ok;             // all float arrays 16-byte and loss_mask 4-byte aligned
+  int keep_vec_ok;        // token_keep and loss_mask 16-byte aligned: 16-token keep stores
   int grid;               // persistent CTAs (sequences are strided over them)
 };
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream);
