@@ -531,6 +531,7 @@ mc_status mc_grpo_masked_loss(const float* logp_policy, const float* logp_behavi
   a.n_clipped = n_clipped;
   a.kl = kl;
   a.Z = reinterpret_cast<long long*>(ws);
+  a.ticket = reinterpret_cast<unsigned int*>(ws + sizeof(long long));
   a.seq_share = reinterpret_cast<float*>(ws + kStatusBytes);
   a.seq_kl = reinterpret_cast<float*>(ws + kStatusBytes + align_up(size_t(B) * sizeof(float), 256));
   a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && aligned(grad_logp, 16) &&

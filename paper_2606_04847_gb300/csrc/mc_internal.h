@@ -156,7 +156,8 @@ struct LossArgs {
   float* seq_loss;
   int32_t* n_clipped;
   float* kl;
-  long long* Z;           // workspace
+  long long* Z;           // workspace (zeroed by the launch, with the ticket after it)
+  unsigned int* ticket;   // workspace: CTAs done, for the last-CTA sum
   float* seq_share;       // workspace [B]
   float* seq_kl;          // workspace [B]
   int vec_ok;

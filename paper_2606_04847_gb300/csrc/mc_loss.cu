@@ -9,12 +9,12 @@
 //            Z = sum_i M_i L_i                                      (Eq. 17)
 //   dL/dlogp_t = M_i / Z (-rho_t A_i [unclipped branch] + beta (1 - e^r))
 //
-// Three launches: (1) one CTA forms Z from the filter's keep / n_tokens;
-// (2) persistent CTAs stride over the sequences, write g_t for every token
-// (16-byte loads and stores, two vectors in flight per thread) and each
-// response's shares of L and of the KL estimate; (3) one CTA sums the shares
-// in a fixed order. All reductions are fixed-order, so results are bitwise
-// reproducible.
+// Two launches: (1) Z from the filter's keep / n_tokens, an exact integer
+// sum over many CTAs; (2) persistent CTAs stride over the sequences, write g_t
+// for every token (16-byte loads and stores, two vectors in flight per
+// thread) and each response's shares of L and of the KL estimate; the last
+// CTA to finish sums the shares in a fixed order. Every floating-point
+// reduction has a fixed order, so results are bitwise reproducible.
 #include "mc_internal.h"
 #include "mc_ptx.cuh"
 
@@ -25,23 +25,20 @@ namespace {
 constexpr int kLossThreads = 256;
 constexpr int kReduceThreads = 1024;
 
+// Z = sum_i M_i L_i over every sequence: an integer sum, so CTAs may add
+// their warps' parts with 64-bit atomics in any order and Z stays exact.
+// (*Z is zeroed on the stream before.) Block 0 also zeroes the clip count.
 __global__ void __launch_bounds__(kReduceThreads) grpo_norm_kernel(const uint8_t* __restrict__ keep,
                                                                    const int32_t* __restrict__ n_tokens, int B,
                                                                    long long* Z, int32_t* n_clipped) {
-  __shared__ long long part[kReduceThreads / 32];
-  long long acc = 0;
-  for (int i = threadIdx.x; i < B; i += blockDim.x)
-    if (keep[i]) acc += n_tokens[i] > 0 ? n_tokens[i] : 0;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  long long v = 0;
+  if (i < B && keep[i]) v = n_tokens[i] > 0 ? n_tokens[i] : 0;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    long long z = 0;
-    for (int w = 0; w < kReduceThreads / 32; ++w) z += part[w];
-    *Z = z;
-    if (n_clipped) *n_clipped = 0;
-  }
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if ((threadIdx.x & 31) == 0 && v != 0)
+    atomicAdd(reinterpret_cast<unsigned long long*>(Z), static_cast<unsigned long long>(v));
+  if (blockIdx.x == 0 && threadIdx.x == 0 && n_clipped) *n_clipped = 0;
 }
 
 struct TokAcc {
@@ -163,51 +160,75 @@ __global__ void __launch_bounds__(kLossThreads) grpo_loss_kernel(LossArgs p) {
     }
     __syncthreads();  // warp_acc is reused by the next sequence
   }
-}
 
-__global__ void __launch_bounds__(kReduceThreads) grpo_final_kernel(const float* __restrict__ seq_share,
-                                                                    const float* __restrict__ seq_kl, int B,
-                                                                    float* loss, float* kl) {
-  __shared__ float part[2][kReduceThreads / 32];
-  float acc = 0.f, acck = 0.f;
-  for (int i = threadIdx.x; i < B; i += blockDim.x) {
-    acc += seq_share[i];
-    acck += seq_kl[i];
+  // The last CTA to finish sums the per-sequence shares in a fixed order
+  // (deterministic): every CTA publishes its shares, then takes a ticket.
+  __shared__ bool last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(p.ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  // Four consecutive shares per thread and step (one 16-byte load from each
+  // 256-byte-aligned workspace array), four partial sums combined in order.
+  float la[4] = {0.f, 0.f, 0.f, 0.f}, ka[4] = {0.f, 0.f, 0.f, 0.f};
+  const int B4 = p.B & ~3;
+#pragma unroll 4
+  for (int i = 4 * threadIdx.x; i < B4; i += 4 * blockDim.x) {
+    const float4 sv = __ldcg(reinterpret_cast<const float4*>(p.seq_share + i));
+    const float4 kv = __ldcg(reinterpret_cast<const float4*>(p.seq_kl + i));
+    la[0] += sv.x;
+    la[1] += sv.y;
+    la[2] += sv.z;
+    la[3] += sv.w;
+    ka[0] += kv.x;
+    ka[1] += kv.y;
+    ka[2] += kv.z;
+    ka[3] += kv.w;
   }
+  if (threadIdx.x < p.B - B4) {
+    la[0] += __ldcg(p.seq_share + B4 + threadIdx.x);
+    ka[0] += __ldcg(p.seq_kl + B4 + threadIdx.x);
+  }
+  float l = (la[0] + la[1]) + (la[2] + la[3]);
+  float k = (ka[0] + ka[1]) + (ka[2] + ka[3]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    acck += __shfl_xor_sync(0xffffffffu, acck, o);
+    l += __shfl_xor_sync(0xffffffffu, l, o);
+    k += __shfl_xor_sync(0xffffffffu, k, o);
   }
   if ((threadIdx.x & 31) == 0) {
-    part[0][threadIdx.x >> 5] = acc;
-    part[1][threadIdx.x >> 5] = acck;
+    warp_acc[threadIdx.x >> 5].s = l;
+    warp_acc[threadIdx.x >> 5].kl = k;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    float l = 0.f, k = 0.f;
-    for (int w = 0; w < kReduceThreads / 32; ++w) {
-      l += part[0][w];
-      k += part[1][w];
+    float lt = 0.f, kt = 0.f;
+    for (int w = 0; w < kLossThreads / 32; ++w) {
+      lt += warp_acc[w].s;
+      kt += warp_acc[w].kl;
     }
-    *loss = l;
-    if (kl) *kl = k;
+    *p.loss = lt;
+    if (p.kl) *p.kl = kt;
   }
 }
 
 }  // namespace
 
 cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream) {
-  grpo_norm_kernel<<<1, kReduceThreads, 0, stream>>>(a.keep, a.n_tokens, a.B, a.Z, a.n_clipped);
-  cudaError_t e = cudaGetLastError();
+  // Z and the ticket counter start at zero.
+  cudaError_t e = cudaMemsetAsync(a.Z, 0, sizeof(long long) + sizeof(unsigned int), stream);
+  if (e != cudaSuccess) return e;
+  grpo_norm_kernel<<<(a.B + kReduceThreads - 1) / kReduceThreads, kReduceThreads, 0, stream>>>(
+      a.keep, a.n_tokens, a.B, a.Z, a.n_clipped);
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int grid = a.B < a.grid ? a.B : a.grid;
   if (a.logp_ref != nullptr)
     grpo_loss_kernel<true><<<grid, kLossThreads, 0, stream>>>(a);
   else
     grpo_loss_kernel<false><<<grid, kLossThreads, 0, stream>>>(a);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  grpo_final_kernel<<<1, kReduceThreads, 0, stream>>>(a.seq_share, a.seq_kl, a.B, a.loss, a.kl);
   return cudaGetLastError();
 }
 
