@@ -57,9 +57,16 @@ def _peaks():
 
 
 def _kernel_source_hash():
+    """Hash of the forward kernel's and its schedule's code, comments and
+    whitespace removed (so that edits to comments keep a capture valid)."""
+    import re
+
     h = hashlib.sha256()
     for f in ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu", "mc_schedule.h"):  # the forward kernel and its schedule
-        h.update(open(os.path.join(ROOT, "paper_2606_04847_gb300", "csrc", f), "rb").read())
+        src = open(os.path.join(ROOT, "paper_2606_04847_gb300", "csrc", f)).read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

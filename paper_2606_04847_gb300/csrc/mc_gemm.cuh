@@ -1,26 +1,29 @@
 // mc_gemm.cuh — persistent warp-specialised tcgen05 GEMM engine for sm_103a.
 //
 // C[m, n] = sum_k A[m, k] B[n, k], bf16 operands, fp32 accumulation in TMEM.
-// The accumulator tile (BM x BN = 128 x 256) is handed to an epilogue functor
-// and never written to memory by the engine itself: the forward turns it into
-// an online log-sum-exp / entropy update, the backward into dZ, the backward
-// GEMMs into plain stores.
+// The accumulator tile (128 x 256, or 256 x 256 with MS = 2) is handed to an
+// epilogue functor and never written to memory by the engine itself: the
+// forward turns it into an online log-sum-exp / entropy update, the backward
+// into dZ, the backward GEMMs into plain stores.
 //
-// CTA = 2 + 4 * MS warps, one CTA per SM (the SMEM ring takes ~194 KB):
-//   warp 0        TMA producer: loads A/B k-blocks (BK = 64) into a 4-stage ring
-//   warp 1        TMEM allocator + MMA issuer (one thread): 4 x tcgen05.mma
-//                 (M=128, N=256, K=16) per k-block into one of two TMEM
-//                 accumulators (2 x 256 fp32 columns = all 512 columns)
+// CTA = 2 + 4 * MS warps, one CTA per SM (the SMEM ring takes 192 KB, plus
+// the epilogue's own staging buffers when it asks for them):
+//   warp 0        TMA producer: loads A/B k-blocks (BK = 64) into the ring
+//                 (4 x 48 KB stages; 3 x 64 KB with MS = 2)
+//   warp 1        TMEM allocator + MMA issuer (one thread): 4 x MS
+//                 tcgen05.mma (M=128, N=256, K=16) per k-block into TMEM
+//                 (2 x 256 fp32 columns = all 512 columns)
 //   warps 2..     epilogue (4 warps per 128-row sub-block): warp w reads TMEM
 //                 lanes 32*(w%4)..+31 of its sub-block, one output row per
 //                 thread, 32 columns per tcgen05.ld
-// The two accumulators let the epilogue of tile j overlap the MMAs of tile
-// j+1 (or, with MS = 2, hold the two 128-row halves of one 256 x 256 tile:
-// see TileCfg). Barriers: full[s]/empty[s] per ring stage, tfull[a]/tempty[a]
-// per accumulator. Every wait is bounded (mbar_wait), and on the way out each
-// role drains what it has in flight (TMA loads, MMAs) before TMEM is freed.
+// With MS = 1 the two 256-column accumulators let the epilogue of tile j
+// overlap the MMAs of tile j+1; with MS = 2 they hold the two 128-row halves
+// of one 256 x 256 tile (see TileCfg). Barriers: full[s]/empty[s] per ring
+// stage, tfull[a]/tempty[a] per accumulator slot. Every wait is bounded
+// (mbar_wait), and on the way out each role drains what it has in flight (TMA
+// loads, MMAs, the epilogue's TMA stores) before TMEM is freed.
 //
-// Work decomposition: the M dimension is cut into BM-row blocks, the N
+// Work decomposition: the M dimension is cut into row blocks, the N
 // dimension into BN-column tiles, and the tiles of one row block into
 // `splits` contiguous ranges. A unit = (row block, range). Units are dealt
 // round-robin to the persistent CTAs (unit u -> CTA u % gridDim.x), so the
@@ -32,9 +35,10 @@
 // Operand layouts: A is [M, K] K-major (A_MN = false) or [K, M] M-major
 // (A_MN = true); B is [N, K] K-major or [K, N] N-major. All tiles use the
 // 128-byte swizzle; TMA boxes are 64 elements (128 B) wide in the contiguous
-// dimension. K-major A: one box {64 k, 128 m}; M-major A: two boxes
-// {64 m, 64 k}; K-major B: one box {64 k, 256 n}; N-major B: four boxes
-// {64 n, 64 k}. Out-of-range rows/columns are zero-filled by TMA.
+// dimension. K-major A: one box {64 k, 128 m} per sub-block; M-major A: two
+// boxes {64 m, 64 k} per sub-block; K-major B: one box {64 k, 256 n}; N-major
+// B: four boxes {64 n, 64 k}. Out-of-range rows/columns are zero-filled by
+// TMA.
 #pragma once
 
 #include <type_traits>
