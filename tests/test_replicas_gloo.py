@@ -34,7 +34,7 @@ def _worker(rank, world, port, results):
 def test_two_replicas_weak_scaling_aggregate():
     world = 2
     port = _free_port()
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:  # no fork of this multi-threaded process
         results = m.dict()
         mp.spawn(_worker, args=(world, port, results), nprocs=world, join=True)
         res = dict(results)
@@ -68,7 +68,7 @@ def _allreduce_worker(rank, world, port, results):
 def test_grad_w_allreduce_sums_over_ranks():
     world = 2
     port = _free_port()
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:  # no fork of this multi-threaded process
         results = m.dict()
         mp.spawn(_allreduce_worker, args=(world, port, results), nprocs=world, join=True)
         res = dict(results)
