@@ -49,9 +49,13 @@ inline int concurrent_units(int sms) { return use_pair_engine() ? sms / 2 : sms;
 // streams W once and keeps its conc / s row blocks of hidden rows in L2, so
 // s is at least the count that holds those rows under kWaveRowBytes. Among
 // the counts allowed, the one with the shortest critical path in tiles,
-// waves(s) x ceil(n_tiles / s); counts within 0.5 % of the best resolve to
-// the fewest splits (fewest W streams).
-constexpr double kWaveRowBytes = 40.0 * (1 << 20);
+// waves(s) x ceil(n_tiles / s); counts within kPathSlack of the best resolve
+// to the fewest splits. W is read from HBM once per wave, so fewer splits
+// (fewer, larger waves) stream it fewer times: under the GPU's power cap the
+// DRAM energy saved buys more SM clock than a slightly longer tail costs.
+// Past ~100 MB of rows per wave the hidden rows no longer stay in L2.
+constexpr double kWaveRowBytes = 80.0 * (1 << 20);
+constexpr double kPathSlack = 1.015;
 
 inline int choose_splits(long long m_blocks, int n_tiles, int conc, int rb, int d) {
   long long lo = static_cast<long long>(std::ceil(double(conc) * rb * d * 2.0 / kWaveRowBytes));
@@ -66,7 +70,7 @@ inline int choose_splits(long long m_blocks, int n_tiles, int conc, int rb, int 
   }
   for (long long s = lo; s <= hi; ++s) {
     const double path = double(ceil_div(m_blocks * s, conc)) * double(ceil_div(n_tiles, s));
-    if (path <= best_path * 1.005) return static_cast<int>(s);
+    if (path <= best_path * kPathSlack) return static_cast<int>(s);
   }
   return static_cast<int>(hi);
 }
