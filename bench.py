@@ -591,8 +591,9 @@ def run_stream(args):
     print(json.dumps(res), flush=True)
 
 
-def _time_calls(fn, launches):
-    fn()
+def _time_calls(fn, launches, warmup=3):
+    for _ in range(warmup):
+        fn()
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record()

@@ -6,11 +6,11 @@
 //         + beta1 1[success_{i,1}] + beta2 1[!success_{i,1} && success_{i,2}]
 //   A_i = (R_i - mean_G R) / (std_G R + eps),  std with divisor G - 1
 //
-// Group sizes dividing 32 (the paper's G = 8 among them): one thread per
-// trajectory, a group's G trajectories on G consecutive lanes of a warp (a
-// group never straddles two warps), its mean and standard deviation formed by
-// xor-shuffle butterflies inside those lanes; a warp reads 32 consecutive
-// trajectory rows. Other group sizes: one thread per group forms the G
+// Group sizes dividing 32 (the paper's G = 8 among them): a group's G
+// trajectories on G consecutive lanes of a warp (a group never straddles two
+// warps), its mean and standard deviation formed by xor-shuffle butterflies
+// inside those lanes; a warp reads 32 consecutive trajectory rows, and each
+// thread handles four rows one block apart. Other group sizes: one thread per group forms the G
 // rewards, then the mean and the standard deviation in two passes.
 #include "mc_internal.h"
 
@@ -74,30 +74,47 @@ __device__ __forceinline__ float trajectory_reward4(const AdvArgs& p, long long 
   return p.alpha * s.x + (1.f - p.alpha) * best + bonus;
 }
 
+// Trajectories per thread in the lanes kernel: thread t of a block handles
+// trajectories base + t + u * blockDim.x, u < kAdvUnroll (whole warps, so
+// whole groups, per u). All of a thread's row loads issue before any reward
+// is formed: four rows' 24 bytes each in flight per thread instead of one.
+constexpr int kAdvUnroll = 4;
+
 template <int G>
 __global__ void __launch_bounds__(kAdvThreads) group_advantage_lanes_kernel(AdvArgs p) {
   static_assert(32 % G == 0, "a group must fit the lanes of one warp");
-  const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
-  const bool live = i < p.n_groups * G;  // whole groups: the tail's dead lanes form dead groups
-  const float r = !live ? 0.f : (p.vec4 ? trajectory_reward4(p, i) : trajectory_reward(p, i));
-  float sum = r;
+  const long long T = p.n_groups * G;
+  const long long base = static_cast<long long>(blockIdx.x) * (blockDim.x * kAdvUnroll) + threadIdx.x;
+  float r[kAdvUnroll];
 #pragma unroll
-  for (int off = G / 2; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-  const float mean = sum / static_cast<float>(G);
-  const float dv = r - mean;
-  float ss = dv * dv;
+  for (int u = 0; u < kAdvUnroll; ++u) {
+    const long long i = base + static_cast<long long>(u) * blockDim.x;
+    // Whole groups: the tail's dead lanes form dead groups.
+    r[u] = i >= T ? 0.f : (p.vec4 ? trajectory_reward4(p, i) : trajectory_reward(p, i));
+  }
 #pragma unroll
-  for (int off = G / 2; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-  if (!live) return;
-  const float sd = G > 1 ? sqrtf(ss / static_cast<float>(G - 1)) : 0.f;
-  if (p.reward) p.reward[i] = r;
-  p.advantage[i] = (G > 1 && sd + p.eps > 0.f) ? dv * (1.f / (sd + p.eps)) : 0.f;
+  for (int u = 0; u < kAdvUnroll; ++u) {
+    const long long i = base + static_cast<long long>(u) * blockDim.x;
+    float sum = r[u];
+#pragma unroll
+    for (int off = G / 2; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    const float mean = sum / static_cast<float>(G);
+    const float dv = r[u] - mean;
+    float ss = dv * dv;
+#pragma unroll
+    for (int off = G / 2; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    if (i >= T) continue;
+    const float sd = G > 1 ? sqrtf(ss / static_cast<float>(G - 1)) : 0.f;
+    if (p.reward) __stcs(p.reward + i, r[u]);
+    __stcs(p.advantage + i, (G > 1 && sd + p.eps > 0.f) ? dv * (1.f / (sd + p.eps)) : 0.f);
+  }
 }
 
 template <int G>
 cudaError_t launch_lanes(const AdvArgs& a, cudaStream_t stream) {
   const long long T = a.n_groups * G;
-  const long long blocks = (T + kAdvThreads - 1) / kAdvThreads;
+  const long long per_block = static_cast<long long>(kAdvThreads) * kAdvUnroll;
+  const long long blocks = (T + per_block - 1) / per_block;
   group_advantage_lanes_kernel<G><<<static_cast<unsigned>(blocks), kAdvThreads, 0, stream>>>(a);
   return cudaGetLastError();
 }
