@@ -674,16 +674,39 @@ def run_next(args):
     res["advantage"] = {}
     for T in (512, 1 << 24):
         K, G = 4, 8
-        gg = torch.Generator(device="cuda").manual_seed(1)
-        scores = torch.rand((T, K), generator=gg, device="cuda") * 2 - 0.5
-        success = (torch.rand((T, K), generator=gg, device="cuda") < 0.3).to(torch.uint8)
-        n_turns = torch.randint(1, K + 1, (T,), generator=gg, device="cuda", dtype=torch.int32)
+        scores, success, n_turns = _advantage_inputs(T, K)
         ms_a = _time_calls(lambda: mc.prime_echo_advantages(scores, success, n_turns, G, 0.75, 0.5, 0.2),
                            args.launches)
         bpt = 5 * K + 4 + 8
         res["advantage"][str(T)] = {"trajectories": T, "turns": K, "group": G, "us": ms_a * 1e3,
                                     "bytes_per_trajectory": bpt, "achieved_gbs": bpt * T / (ms_a / 1e3) / 1e9}
     print(json.dumps(res), flush=True)
+
+
+def _advantage_inputs(T, K):
+    """Seeded per-turn scores in [-0.5, 1.5), success flags (30 % set) and turn
+    counts in [1, K] for T trajectories, on the GPU."""
+    gg = torch.Generator(device="cuda").manual_seed(1)
+    scores = torch.rand((T, K), generator=gg, device="cuda") * 2 - 0.5
+    success = (torch.rand((T, K), generator=gg, device="cuda") < 0.3).to(torch.uint8)
+    n_turns = torch.randint(1, K + 1, (T,), generator=gg, device="cuda", dtype=torch.int32)
+    return scores, success, n_turns
+
+
+def run_advantage(args):
+    """--case advantage: the reward + group advantage on 2^24 four-turn
+    trajectories in groups of 8, `--launches` calls (for ncu captures), with
+    the CUDA-event time per call."""
+    from paper_2606_04847_gb300 import mc
+
+    torch.cuda.set_device(0)
+    T, K, G = 1 << 24, 4, 8
+    scores, success, n_turns = _advantage_inputs(T, K)
+    ms = _time_calls(lambda: mc.prime_echo_advantages(scores, success, n_turns, G, 0.75, 0.5, 0.2),
+                     args.launches)
+    bpt = 5 * K + 4 + 8
+    print(json.dumps({"case": "advantage", "trajectories": T, "launches": args.launches, "us": ms * 1e3,
+                      "bytes_per_trajectory": bpt, "achieved_gbs": bpt * T / (ms / 1e3) / 1e9}))
 
 
 def run_case(args):
@@ -697,6 +720,8 @@ def run_case(args):
         return run_stream(args)
     if args.case == "next":
         return run_next(args)
+    if args.case == "advantage":
+        return run_advantage(args)
     torch.cuda.set_device(0)
     if not os.path.exists(mc.lib_path()):
         mcbuild.build()
@@ -781,7 +806,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-rows", type=int, default=384)
     ap.add_argument("--ref-rows", type=int, default=64)
-    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream", "next"], default="step",
+    ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream", "next", "advantage"],
+                    default="step",
                     help="profiling aid: run one call of the path --launches times")
     ap.add_argument("--rows", type=int, default=0, help="--case: tokens to use (0 = the whole batch)")
     ap.add_argument("--launches", type=int, default=2)

@@ -476,7 +476,7 @@ mc_status mc_seq_ratio_filter(const float* logp_policy, const float* logp_behavi
   a.vec_ok = aligned(logp_policy, 16) && aligned(logp_behaviour, 16) && (!token_ratio || aligned(token_ratio, 16)) &&
              (!loss_mask || aligned(loss_mask, 4));
   a.keep_vec_ok = aligned(token_keep, 16) && (!loss_mask || aligned(loss_mask, 16));
-  a.grid = 16 * sms;
+  a.grid = mc::filter_ctas_per_sm() * sms;
   cudaError_t e = mc::launch_filter(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "filter launch");
   return MC_OK;

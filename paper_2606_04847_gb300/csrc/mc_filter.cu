@@ -1,17 +1,18 @@
 // mc_filter.cu — per-sequence importance-ratio statistics and the MirrorPop
 // keep-mask (§4.5.2, Eq. 18-21), plus per-token ratios (Eq. 4).
 //
-// Persistent CTAs (16 per SM, 128 threads each) stride over the sequences, one
-// sequence at a time per CTA. Each thread walks its share of the sequence's packed tokens
-// with 16-byte loads (4 tokens of logp_policy / logp_behaviour, 4 mask bytes;
-// two vectors in flight), accumulates sum(log rho), sum(|log rho|) and the
-// count over loss-masked tokens, and writes rho = exp(log rho) on the way
-// (streaming stores). Warp shuffles then
-// a shared-memory step reduce the three sums in a fixed order (deterministic
-// for a given launch shape). Thread 0 forms the statistics and the masks; a
-// second sweep writes token_keep once keep_i is known, 16 tokens per 16-byte
-// load of the mask and store. The kernel is HBM-
-// bound: 4 + 4 + 1 bytes read and up to 4 + 1 bytes written per token.
+// Persistent CTAs of 128 threads, as many as the SMs keep resident at once (12
+// per SM at the kernel's 37 registers: one wave, no late second wave at low
+// occupancy), stride over the sequences, one sequence at a time per CTA. Each
+// thread walks its share of the sequence's packed tokens with 16-byte loads
+// (4 tokens of logp_policy / logp_behaviour, 4 mask bytes; two vectors in
+// flight), accumulates sum(log rho), sum(|log rho|) and the count over
+// loss-masked tokens, and writes rho = exp(log rho) on the way (streaming
+// stores). Warp shuffles then a shared-memory step reduce the three sums in a
+// fixed order (deterministic for a given launch shape). Thread 0 forms the
+// statistics and the masks; a second sweep writes token_keep once keep_i is
+// known, 16 tokens per 16-byte load of the mask and store. The kernel is
+// HBM-bound: 4 + 4 + 1 bytes read and up to 4 + 1 bytes written per token.
 #include "mc_internal.h"
 #include "mc_ptx.cuh"
 
@@ -172,6 +173,19 @@ __global__ void selftest_wait_kernel(int32_t* dev_status, uint64_t timeout_ns) {
 }
 
 }  // namespace
+
+int filter_ctas_per_sm() {
+  static const int n = [] {
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, seq_filter_kernel, kFilterThreads, 0) != cudaSuccess ||
+        b < 1) {
+      cudaGetLastError();  // clear the failed query, so the launch check after it does not report it
+      b = 1;
+    }
+    return b;
+  }();
+  return n;
+}
 
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream) {
   if (a.B <= 0) return cudaSuccess;

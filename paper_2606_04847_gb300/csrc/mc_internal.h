@@ -137,6 +137,9 @@ struct FilterArgs {
   int grid;               // persistent CTAs (sequences are strided over them)
 };
 cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream);
+// CTAs of the filter kernel one SM keeps resident (from its register and
+// thread counts, queried once): a grid of SMs x this runs in a single wave.
+int filter_ctas_per_sm();
 
 struct LossArgs {
   const float* logp_policy;
