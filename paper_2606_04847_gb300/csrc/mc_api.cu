@@ -366,6 +366,10 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
   sa.idx = idx;
   sa.count = count;
   sa.hc = hc;
+  // The slab offsets of the row selection live at the start of the gathered-
+  // rows region: selection finishes with them before the gather writes it
+  // (n_pad * d * 2 bytes, far more than the ceil(N / 1024) * 4 they take).
+  sa.slab = reinterpret_cast<int32_t*>(hc);
   sa.ws_status = ws_status;
   sa.grid = sms * 8;
   if ((e = mc::launch_select_gather(sa, s)) != cudaSuccess) return cuda_fail(e, "row selection launch");

@@ -40,50 +40,99 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 // ---------------------------------------------------------------- stage 0
 
-// One CTA: ordered compaction of the rows with a nonzero effective upstream
-// gradient. Block-wide exclusive scan per 1024-row slab (warp ballots, then a
-// warp scan of the 32 warp counts).
-__global__ void __launch_bounds__(kSelectThreads) select_rows_kernel(
+// Ordered compaction of the rows with a nonzero effective upstream gradient,
+// in three launches over slabs of kSelectThreads rows: (1) each slab's count
+// of selected rows (and the target range check), (2) one CTA turns the counts
+// into exclusive offsets and writes the total, (3) each slab writes its rows'
+// indices from its offset, in row order (a block scan of warp ballots). No CTA
+// waits on another.
+__device__ __forceinline__ int select_flag(const uint8_t* __restrict__ row_keep, const float* __restrict__ g,
+                                           const float* __restrict__ gh, const int32_t* __restrict__ targets,
+                                           int V, long long t, bool& bad_target) {
+  const int y = targets[t];
+  const bool yok = y >= 0 && y < V;
+  bad_target |= !yok;
+  const bool live = g[t] != 0.f || (gh != nullptr && gh[t] != 0.f);
+  return (yok && live && (row_keep == nullptr || row_keep[t] != 0)) ? 1 : 0;
+}
+
+__global__ void __launch_bounds__(kSelectThreads) select_count_kernel(
     const uint8_t* __restrict__ row_keep, const float* __restrict__ g, const float* __restrict__ gh,
-    const int32_t* __restrict__ targets, int V, long long N, int32_t* __restrict__ idx, int32_t* count,
-    int32_t* status) {
+    const int32_t* __restrict__ targets, int V, long long N, int32_t* __restrict__ slab, int32_t* status) {
+  const long long t = static_cast<long long>(blockIdx.x) * kSelectThreads + threadIdx.x;
+  bool bad = false;
+  const int f = t < N ? select_flag(row_keep, g, gh, targets, V, t, bad) : 0;
+  const int n = __syncthreads_count(f);
+  const int any_bad = __syncthreads_or(bad);
+  if (threadIdx.x == 0) {
+    slab[blockIdx.x] = n;
+    if (any_bad) atomicOr(status, MC_DEV_TARGET_RANGE);
+  }
+}
+
+// Exclusive prefix sum of the slab counts, in place, in chunks of
+// kSelectThreads; *count = the total.
+__global__ void __launch_bounds__(kSelectThreads) select_scan_kernel(int32_t* __restrict__ slab, long long nslabs,
+                                                                     int32_t* count) {
   __shared__ int warp_off[kSelectThreads / 32];
-  __shared__ int slab_total;
+  __shared__ int chunk_total;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int base = 0;
-  bool bad_target = false;
-  for (long long start = 0; start < N; start += kSelectThreads) {
-    const long long t = start + tid;
-    int f = 0;
-    if (t < N) {
-      const int y = targets[t];
-      const bool yok = y >= 0 && y < V;
-      bad_target |= !yok;
-      const bool live = g[t] != 0.f || (gh != nullptr && gh[t] != 0.f);
-      f = (yok && live && (row_keep == nullptr || row_keep[t] != 0)) ? 1 : 0;
+  for (long long s0 = 0; s0 < nslabs; s0 += kSelectThreads) {
+    const long long s = s0 + tid;
+    const int c = s < nslabs ? slab[s] : 0;
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
     }
-    const unsigned bal = __ballot_sync(0xffffffffu, f);
-    const int in_warp = __popc(bal & ((1u << lane) - 1u));
-    if (lane == 0) warp_off[warp] = __popc(bal);
+    if (lane == 31) warp_off[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-      const int c = warp_off[lane];
-      int incl = c;
+      const int w = warp_off[lane];
+      int wi = w;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const int n = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += n;
+        const int n = __shfl_up_sync(0xffffffffu, wi, o);
+        if (lane >= o) wi += n;
       }
-      warp_off[lane] = incl - c;
-      if (lane == 31) slab_total = incl;
+      warp_off[lane] = wi - w;
+      if (lane == 31) chunk_total = wi;
     }
     __syncthreads();
-    if (f) idx[base + warp_off[warp] + in_warp] = static_cast<int32_t>(t);
-    base += slab_total;
+    if (s < nslabs) slab[s] = base + warp_off[warp] + incl - c;
+    base += chunk_total;
     __syncthreads();
   }
-  if (__syncthreads_or(bad_target) && tid == 0) atomicOr(status, MC_DEV_TARGET_RANGE);
   if (tid == 0) *count = base;
+}
+
+__global__ void __launch_bounds__(kSelectThreads) select_write_kernel(
+    const uint8_t* __restrict__ row_keep, const float* __restrict__ g, const float* __restrict__ gh,
+    const int32_t* __restrict__ targets, int V, long long N, const int32_t* __restrict__ slab,
+    int32_t* __restrict__ idx) {
+  __shared__ int warp_off[kSelectThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const long long t = static_cast<long long>(blockIdx.x) * kSelectThreads + tid;
+  bool bad = false;
+  const int f = t < N ? select_flag(row_keep, g, gh, targets, V, t, bad) : 0;
+  const unsigned bal = __ballot_sync(0xffffffffu, f);
+  const int in_warp = __popc(bal & ((1u << lane) - 1u));
+  if (lane == 0) warp_off[warp] = __popc(bal);
+  __syncthreads();
+  if (warp == 0) {
+    const int c = warp_off[lane];
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    warp_off[lane] = incl - c;
+  }
+  __syncthreads();
+  if (f) idx[slab[blockIdx.x] + warp_off[warp] + in_warp] = static_cast<int32_t>(t);
 }
 
 // Hc[j] = H[idx[j]] for j < count, zero rows up to the next multiple of 256
@@ -349,10 +398,22 @@ __global__ void status_merge(const int32_t* ws_status, int32_t* dev_status) {
 }  // namespace
 
 cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
-  select_rows_kernel<<<1, kSelectThreads, 0, stream>>>(a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V,
-                                                       a.N, a.idx, a.count, a.ws_status);
+  const long long nslabs = (a.N + kSelectThreads - 1) / kSelectThreads;
+  if (nslabs > 0) {
+    select_count_kernel<<<static_cast<unsigned>(nslabs), kSelectThreads, 0, stream>>>(
+        a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V, a.N, a.slab, a.ws_status);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  select_scan_kernel<<<1, kSelectThreads, 0, stream>>>(a.slab, nslabs, a.count);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (nslabs > 0) {
+    select_write_kernel<<<static_cast<unsigned>(nslabs), kSelectThreads, 0, stream>>>(
+        a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V, a.N, a.slab, a.idx);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   const int row_vec = a.d * 2 / 16;
   gather_rows_kernel<<<a.grid, 256, 0, stream>>>(static_cast<const uint4*>(a.hidden), row_vec, a.idx, a.count,
                                                  static_cast<uint4*>(a.hc));

@@ -50,6 +50,7 @@ struct SelectArgs {
   int d, V;
   int32_t* idx;           // workspace: [N] selected original rows, ascending
   int32_t* count;         // workspace: number selected
+  int32_t* slab;          // workspace: [ceil(N / 1024)] per-slab offsets (any region the gather writes later)
   void* hc;               // workspace: bf16 [n_pad, d] gathered hidden rows
   int32_t* ws_status;
   int grid;
