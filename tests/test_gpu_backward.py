@@ -207,3 +207,30 @@ def test_zero_rows():
     out = mc.token_logprobs_bwd(h, w, y, z, None, z)
     torch.cuda.synchronize()
     assert out["grad_hidden"].shape == (0, 64) and not out["grad_w"].any()
+
+
+def test_out_of_range_targets_are_skipped_and_flagged():
+    """Targets outside [0, V) in two different 1,024-row selection slabs: the
+    row selection sets MC_DEV_TARGET_RANGE and leaves those rows out (zero
+    gradient, their NaN lse never read); every other row matches the oracle
+    with those rows' upstream gradient zeroed."""
+    wl, g, ge = setup(2100, 64, 700, seed=22)
+    y_bad = wl.targets.clone()
+    y_bad[5] = 700
+    y_bad[1500] = -1
+    h, w = wl.hidden.cuda(), wl.w_vocab.cuda()
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    fw = mc.token_logprobs(h, w, y_bad.cuda())
+    out = mc.token_logprobs_bwd(h, w, y_bad.cuda(), fw["lse"], fw["entropy"], g.cuda(), ge.cuda(), dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & mc.MC_DEV_TARGET_RANGE
+    gh = out["grad_hidden"]
+    assert not gh[5].any() and not gh[1500].any()
+    g0, ge0 = g.clone(), ge.clone()
+    g0[[5, 1500]] = 0.0
+    ge0[[5, 1500]] = 0.0
+    y_ok = y_bad.clone()
+    y_ok[[5, 1500]] = 0
+    ref = oracle.token_logprobs_bwd(wl.hidden, wl.w_vocab, y_ok, g0, ge0)
+    assert rel_fro(np_(gh.float()), ref["grad_hidden"]) <= TOL_GRAD
+    assert rel_fro(np_(out["grad_w"]), ref["grad_w"]) <= TOL_GRAD
