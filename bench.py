@@ -604,9 +604,32 @@ def _time_calls(fn, launches, warmup=3):
     return a.elapsed_time(b) / launches
 
 
+def _time_graph(fn, launches, warmup=3):
+    """Per-call GPU time of `launches` calls of fn captured into one CUDA graph
+    and replayed: the kernels alone, without the host's per-call launch gaps
+    (the calls must be capturable: stream-ordered, no synchronisation)."""
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        for _ in range(launches):
+            fn()
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / launches
+
+
 def run_next(args):
     """Measurements of the rows beyond the main path (CUDA events over
-    --launches calls each), one JSON line:
+    --launches calls each, after three untimed; the launch-bound merge and
+    the 512-trajectory advantage from a CUDA-graph replay of those calls, with
+    their eager per-call times beside), one JSON line:
     * the masked GRPO loss with the beta * KL term (reference log-probs) on
       64M tokens in 16,384 sequences: HBM GB/s for 4 + 4 + 4 + 1 B read and
       4 B written per token;
@@ -661,11 +684,13 @@ def run_next(args):
 
     merged = mc.merge_logprob_states(states)
     ms_s = _time_calls(shard_calls, args.launches)
-    ms_m = _time_calls(lambda: mc.merge_logprob_states(states, out=merged), args.launches)
+    ms_m_eager = _time_calls(lambda: mc.merge_logprob_states(states, out=merged), args.launches)
+    ms_m = _time_graph(lambda: mc.merge_logprob_states(states, out=merged), args.launches)
     flop = 2.0 * Nt * d * V
     res["sharded_forward"] = {"tokens": Nt, "slices": P, "ms_slices": ms_s, "tflops": flop / (ms_s / 1e3) / 1e12,
                               "frac_of_sustained": flop / (ms_s / 1e3) / 1e12 / peaks["bf16_sustained"],
-                              "merge_ms": ms_m, "merge_bytes_per_token": 16 * P + 12,
+                              "merge_ms": ms_m, "merge_ms_eager_call": ms_m_eager,
+                              "merge_bytes_per_token": 16 * P + 12,
                               "merge_gbs": (16 * P + 12) * Nt / (ms_m / 1e3) / 1e9}
     del wl, h, w, y, states, ws, slices, merged
     torch.cuda.empty_cache()
@@ -675,11 +700,14 @@ def run_next(args):
     for T in (512, 1 << 24):
         K, G = 4, 8
         scores, success, n_turns = _advantage_inputs(T, K)
-        ms_a = _time_calls(lambda: mc.prime_echo_advantages(scores, success, n_turns, G, 0.75, 0.5, 0.2),
-                           args.launches)
+        call = lambda: mc.prime_echo_advantages(scores, success, n_turns, G, 0.75, 0.5, 0.2)  # noqa: E731
+        ms_eager = _time_calls(call, args.launches)
+        # Small batches are launch-bound: their kernel time comes from a graph replay.
+        ms_a = _time_graph(call, args.launches) if T <= (1 << 16) else ms_eager
         bpt = 5 * K + 4 + 8
         res["advantage"][str(T)] = {"trajectories": T, "turns": K, "group": G, "us": ms_a * 1e3,
-                                    "bytes_per_trajectory": bpt, "achieved_gbs": bpt * T / (ms_a / 1e3) / 1e9}
+                                    "us_eager_call": ms_eager * 1e3, "bytes_per_trajectory": bpt,
+                                    "achieved_gbs": bpt * T / (ms_a / 1e3) / 1e9}
     print(json.dumps(res), flush=True)
 
 
