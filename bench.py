@@ -344,8 +344,11 @@ def run_ours(args):
     torch.cuda.synchronize()
     eager_ms = probe[0].elapsed_time(probe[1])
     use_graph = args.graph == "on" or (args.graph == "auto" and eager_ms < 2.0)
+    graph_launches = 0
     if use_graph:
+        l_cap = mc.kernel_launches()
         capture("resident", resident)
+        graph_launches = mc.kernel_launches() - l_cap  # kernels in one step's graphs (counted at capture)
         for _ in range(args.warmup):
             flt = step()
         torch.cuda.synchronize()
@@ -362,12 +365,17 @@ def run_ours(args):
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
+    l_timed = mc.kernel_launches()
     t_start.record(stream)
     for i in range(args.steps):
         if flush_buf is not None:
             flush_buf.fill_(i & 0xFF)
         step(record=True)
     t_end.record(stream)
+    # libmc's own count of the kernels it enqueued in the timed steps; graph
+    # replays bypass the library's host code, so there it is the kernels
+    # captured into one step's graphs times the steps.
+    gpu_launches = graph_launches * args.steps if use_graph else mc.kernel_launches() - l_timed
     torch.cuda.synchronize()
     _barrier(world)
     clk = clocks.stop()
@@ -496,8 +504,6 @@ def run_ours(args):
                "sample": f"first {rows} packed tokens of the workload (one sequence slice): fp64 forward over "
                          f"V={V}, filter, backward; {secs:.1f} s"}
 
-    # forward + finalize; filter; select, gather, dZ, dH, dW (one row chunk)
-    launches_per_step = 2 + 1 + (5 if has_bwd else 0)
     if rank == 0:
         line = {
             "metric": METRIC if has_bwd else METRIC_FWD,
@@ -527,7 +533,9 @@ def run_ours(args):
             "ms_by_call": {"forward": t_fwd, "filter": t_flt, "backward": t_bwd},
             "clocks": clk,
             "e2e": e2e,
-            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches": gpu_launches,
+            "gpu_launches_source": "libmc launch counter (mc_kernel_launches) over the timed steps" +
+                                   (" (graph replays: kernels captured per step x steps)" if use_graph else ""),
             "roofline": {"bound": "tensor", "kernel": "forward (tcgen05 projection + online log-softmax)",
                          "achieved": achieved, "peak": peak_tf, "unit": "TFLOP/s", "frac": achieved / peak_tf,
                          "peak_source": f"{peaks['source']} bf16 {peak_kind}", "traffic": traffic,

@@ -62,6 +62,12 @@ const char* mc_status_string(mc_status s);
 const char* mc_last_cuda_error(void);
 /* ABI version: (major << 16) | minor. */
 int32_t mc_version(void);
+/* Kernels this library has enqueued in this process since it was loaded, over
+ * every entry point and thread (a relaxed atomic counter). For launch
+ * accounting: the difference across a region of calls is the number of
+ * kernels those calls launched. Calls captured into a CUDA graph count once,
+ * at capture, not at each replay. */
+uint64_t mc_kernel_launches(void);
 
 /* ------------------------------------------------------------------------
  * Forward: per-token target log-prob, entropy and log-sum-exp.

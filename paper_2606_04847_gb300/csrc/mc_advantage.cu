@@ -116,7 +116,7 @@ cudaError_t launch_lanes(const AdvArgs& a, cudaStream_t stream) {
   const long long per_block = static_cast<long long>(kAdvThreads) * kAdvUnroll;
   const long long blocks = (T + per_block - 1) / per_block;
   group_advantage_lanes_kernel<G><<<static_cast<unsigned>(blocks), kAdvThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace
@@ -134,7 +134,7 @@ cudaError_t launch_group_advantage(const AdvArgs& a, cudaStream_t stream) {
   }
   const long long blocks = (a.n_groups + kAdvThreads - 1) / kAdvThreads;
   group_advantage_kernel<<<static_cast<unsigned>(blocks), kAdvThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace mc

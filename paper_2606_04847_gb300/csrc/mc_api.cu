@@ -173,6 +173,13 @@ BwdLayout bwd_layout(int64_t N, int32_t d) {
 
 }  // namespace
 
+namespace mc {
+namespace {
+std::atomic<unsigned long long> g_kernel_launches{0};
+}  // namespace
+void note_launches(unsigned n) { g_kernel_launches.fetch_add(n, std::memory_order_relaxed); }
+}  // namespace mc
+
 extern "C" {
 
 const char* mc_status_string(mc_status s) {
@@ -192,7 +199,9 @@ const char* mc_status_string(mc_status s) {
 
 const char* mc_last_cuda_error(void) { return g_last_cuda_error.c_str(); }
 
-int32_t mc_version(void) { return (1 << 16) | 0; }
+int32_t mc_version(void) { return (1 << 16) | 1; }
+
+uint64_t mc_kernel_launches(void) { return mc::g_kernel_launches.load(std::memory_order_relaxed); }
 
 size_t mc_token_logprobs_workspace_size(int64_t N, int32_t d, int32_t V) {
   if (!valid_common(N, d, V, 1.f)) return 0;

@@ -388,7 +388,7 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
   kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(ta, tb, sch, ep, timeout_ns, status);
-  return cudaGetLastError();
+  return launched();
 }
 
 __global__ void status_merge(const int32_t* ws_status, int32_t* dev_status) {
@@ -402,22 +402,22 @@ cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
   if (nslabs > 0) {
     select_count_kernel<<<static_cast<unsigned>(nslabs), kSelectThreads, 0, stream>>>(
         a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V, a.N, a.slab, a.ws_status);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launched();
     if (e != cudaSuccess) return e;
   }
   select_scan_kernel<<<1, kSelectThreads, 0, stream>>>(a.slab, nslabs, a.count);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launched();
   if (e != cudaSuccess) return e;
   if (nslabs > 0) {
     select_write_kernel<<<static_cast<unsigned>(nslabs), kSelectThreads, 0, stream>>>(
         a.row_keep, a.grad_logp, a.grad_entropy, a.targets, a.V, a.N, a.slab, a.idx);
-    e = cudaGetLastError();
+    e = launched();
     if (e != cudaSuccess) return e;
   }
   const int row_vec = a.d * 2 / 16;
   gather_rows_kernel<<<a.grid, 256, 0, stream>>>(static_cast<const uint4*>(a.hidden), row_vec, a.idx, a.count,
                                                  static_cast<uint4*>(a.hc));
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
@@ -536,7 +536,7 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
 cudaError_t launch_status_merge(const int32_t* ws_status, int32_t* dev_status, cudaStream_t stream) {
   if (dev_status == nullptr) return cudaSuccess;
   status_merge<<<1, 1, 0, stream>>>(ws_status, dev_status);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace mc

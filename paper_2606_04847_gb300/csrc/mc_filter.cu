@@ -191,12 +191,12 @@ cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream) {
   if (a.B <= 0) return cudaSuccess;
   const int grid = a.B < a.grid ? a.B : a.grid;
   seq_filter_kernel<<<grid, kFilterThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream) {
   selftest_wait_kernel<<<1, 32, 0, stream>>>(dev_status, timeout_ns);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace mc

@@ -243,7 +243,7 @@ cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdEpi
   const int units = sch.m_blocks * sch.splits;
   const int grid = units < a.grid ? units : a.grid;
   kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_merge_states(const float* states, int P, long long N, float* logp, float* entropy, float* lse,
@@ -253,7 +253,7 @@ cudaError_t launch_merge_states(const float* states, int P, long long N, float* 
   const long long blocks = (N + threads - 1) / threads;
   merge_states_kernel<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
       reinterpret_cast<const float4*>(states), P, N, logp, entropy, lse, dev_status);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
@@ -293,7 +293,7 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
     fwd_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
         a.targets, a.N, a.V, a.splits, a.n_pad, a.part, a.zy, a.logp, a.entropy, a.lse, a.ws_status,
         a.dev_status);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace mc

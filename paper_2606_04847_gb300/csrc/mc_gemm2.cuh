@@ -23,6 +23,7 @@
 #pragma once
 
 #include "mc_gemm.cuh"
+#include "mc_internal.h"
 
 namespace mc {
 
@@ -293,7 +294,9 @@ cudaError_t run_gemm_pair(const CUtensorMap& ta, const CUtensorMap& tb, const Sc
   const int clusters = static_cast<int>(units < max_clusters ? units : max_clusters);
   if (clusters <= 0) return cudaSuccess;
   cfg.gridDim = dim3(static_cast<unsigned>(2 * clusters), 1, 1);
-  return cudaLaunchKernelEx(&cfg, kern, ta, tb, sch, ep, timeout_ns, status);
+  e = cudaLaunchKernelEx(&cfg, kern, ta, tb, sch, ep, timeout_ns, status);
+  if (e == cudaSuccess) note_launches();
+  return e;
 }
 
 }  // namespace mc

@@ -9,6 +9,16 @@
 
 namespace mc {
 
+// Launch accounting: every kernel the library enqueues is counted (a
+// process-wide relaxed atomic, read through mc_kernel_launches()).
+void note_launches(unsigned n = 1);
+// After a kernel launch: its error status, counting the launch if it was enqueued.
+inline cudaError_t launched() {
+  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) note_launches();
+  return e;
+}
+
 // Forward: persistent tcgen05 kernel (online log-softmax epilogue) followed by
 // the per-row merge of the split partials.
 struct FwdArgs {

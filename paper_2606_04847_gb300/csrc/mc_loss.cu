@@ -222,14 +222,14 @@ cudaError_t launch_grpo_loss(const LossArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   grpo_norm_kernel<<<(a.B + kReduceThreads - 1) / kReduceThreads, kReduceThreads, 0, stream>>>(
       a.keep, a.n_tokens, a.B, a.Z, a.n_clipped);
-  e = cudaGetLastError();
+  e = launched();
   if (e != cudaSuccess) return e;
   const int grid = a.B < a.grid ? a.B : a.grid;
   if (a.logp_ref != nullptr)
     grpo_loss_kernel<true><<<grid, kLossThreads, 0, stream>>>(a);
   else
     grpo_loss_kernel<false><<<grid, kLossThreads, 0, stream>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace mc

@@ -42,6 +42,7 @@ SIGNATURES = {
     "mc_status_string": (ctypes.c_char_p, [_I32]),
     "mc_last_cuda_error": (ctypes.c_char_p, []),
     "mc_version": (_I32, []),
+    "mc_kernel_launches": (ctypes.c_uint64, []),
     "mc_token_logprobs_workspace_size": (_SZ, [_I64, _I32, _I32]),
     "mc_token_logprobs": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _SZ, _P, _P]),
     "mc_token_logprobs_noalloc": (_I32, [_P, _P, _P, _I64, _I32, _I32, _F, _P, _P, _P, _P, _P]),
@@ -138,6 +139,11 @@ def _ws(t: torch.Tensor, device) -> torch.Tensor:
 def version() -> tuple:
     v = lib().mc_version()
     return (v >> 16, v & 0xFFFF)
+
+
+def kernel_launches() -> int:
+    """Kernels libmc has enqueued in this process so far (mc_kernel_launches)."""
+    return int(lib().mc_kernel_launches())
 
 
 def forward_workspace_size(N: int, d: int, V: int) -> int:

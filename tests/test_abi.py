@@ -89,6 +89,19 @@ def test_forward_argument_checks(L):
     assert fwd(L, N=0) == 0  # nothing to do
 
 
+def test_host_detected_errors_queue_no_kernels(L):
+    """Calls rejected on the host (bad sizes, pointers, workspaces) launch
+    nothing: the library's launch counter does not move."""
+    before = L.mc_kernel_launches()
+    assert fwd(L, N=-1) == INVALID
+    assert fwd(L, d=100) == INVALID
+    assert fwd(L, ws=None) == WORKSPACE
+    assert fwd(L, N=0) == 0
+    assert bwd(L, d=100) == INVALID
+    assert bwd(L, ws_bytes=100) == WORKSPACE
+    assert L.mc_kernel_launches() == before
+
+
 def test_forward_without_gpu_reports_device_error(L):
     import torch
 
