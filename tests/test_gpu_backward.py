@@ -95,6 +95,17 @@ def test_single_entry_vocabulary_has_zero_gradient():
     assert out["grad_hidden"].float().abs().max() < 1e-6 and out["grad_w"].abs().max() < 1e-6
 
 
+def test_long_hidden_8192():
+    """d = 8192: 128 k-blocks per dZ tile and a 32-tile grad_hidden output
+    row (128-row tiles: 300 rows), V = 600."""
+    check(*setup(300, 8192, 600, seed=24))
+
+
+def test_wide_tile_dz_long_hidden():
+    """256-row dZ tiles at d = 8192 (4200 rows = 16 blocks + 104), V = 300."""
+    check(*setup(4200, 8192, 300, seed=25))
+
+
 def test_wide_tile_dz_producer():
     """>= 4096 kept rows: the dZ producer runs 256-row tiles (4500 rows =
     17 blocks + 148), with the entropy term and temperature."""

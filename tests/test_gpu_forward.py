@@ -3,7 +3,7 @@
 Sizes span several 128-row blocks and 256-column vocabulary tiles, with
 ragged tails in both, the tiny config at full size, and the edge cases:
 N = 1, V not a multiple of the tile, V < one tile, targets at 0 and V-1,
-peaked softmax (low entropy), temperature, d = 64 and d = 5120.
+peaked softmax (low entropy), temperature, d from 64 to 8192.
 """
 
 import math
@@ -43,6 +43,8 @@ def test_config1_tiny_full_size():
     (129, 256, 200),         # V smaller than one tile
     (520, 512, 151936 // 16),  # 9496 = 37 tiles + 24 columns
     (257, 5120, 1024),       # the 27B-class hidden size
+    (130, 6144, 777),        # 96 k-blocks per tile
+    (300, 8192, 1000),       # 128 k-blocks per tile
 ])
 def test_ragged_shapes(N, d, V):
     spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=d, V=V)
@@ -55,6 +57,13 @@ def test_wide_tiles_ragged(inv_temp):
     blocks + 148), a vocabulary tail of 184 columns."""
     spec = workloads.spec_for(1, n_seqs=1, len_lo=4500, len_hi=4500, d=256, V=3000)
     run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
+
+
+def test_wide_tiles_long_hidden():
+    """256-row tiles with d = 8192 (128 k-blocks through the 3-stage ring per
+    tile): 4200 rows = 16 blocks + 104, V = 300 (a 44-column tail)."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=4200, len_hi=4200, d=8192, V=300, seed=23)
+    run_and_compare(workloads.build(spec, "cpu"))
 
 
 def test_wide_tiles_tiny_vocabulary_single_k_block():
