@@ -95,6 +95,12 @@ def test_single_entry_vocabulary_has_zero_gradient():
     assert out["grad_hidden"].float().abs().max() < 1e-6 and out["grad_w"].abs().max() < 1e-6
 
 
+def test_million_entry_vocabulary():
+    """V = 1,000,003: dZ rows of 2 MB, grad_hidden's K loop over 15,625
+    k-blocks (256-row tiles), 3,907 grad_w row tiles; 64 rows, d = 64."""
+    check(*setup(64, 64, 1_000_003, seed=27))
+
+
 def test_long_hidden_8192():
     """d = 8192: 128 k-blocks per dZ tile and a 32-tile grad_hidden output
     row (128-row tiles: 300 rows), V = 600."""

@@ -59,6 +59,13 @@ def test_wide_tiles_ragged(inv_temp):
     run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
 
 
+def test_million_entry_vocabulary():
+    """V = 1,000,003 (3,907 tiles, a 3-column tail; the maximum 16 splits per
+    row block) on 64 rows, d = 64."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=64, len_hi=64, d=64, V=1_000_003, seed=26)
+    run_and_compare(workloads.build(spec, "cpu"))
+
+
 def test_wide_tiles_long_hidden():
     """256-row tiles with d = 8192 (128 k-blocks through the 3-stage ring per
     tile): 4200 rows = 16 blocks + 104, V = 300 (a 44-column tail)."""
