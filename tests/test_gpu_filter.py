@@ -135,3 +135,12 @@ def test_forward_then_filter_tiny_config():
     got, want = np_(out["keep"]).astype(bool), ref["keep"].astype(bool)
     assert not np.any((got != want) & (np.abs(ref["abs_mean"] - delta) > band))
     assert 0 < want.sum() < wl.B or True  # informational: tiny config threshold sits inside the spread
+
+
+def test_many_tiny_sequences():
+    """100,003 sequences of 0-5 tokens (most shorter than one 16-byte vector,
+    many empty): every persistent CTA strides over dozens of sequences, and
+    the head / vector / tail split of each sequence is exercised at every
+    offset."""
+    lens = torch.randint(0, 6, (100_003,), generator=torch.Generator().manual_seed(11)).tolist()
+    compare(*make(lens, seed=12, mask_p=0.8), 0.1, 0.1)

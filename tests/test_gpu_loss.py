@@ -131,3 +131,11 @@ def test_chain_forward_filter_loss_backward_tiny():
     ref_bw = oracle.token_logprobs_bwd(wl.hidden, wl.w_vocab, wl.targets, ref_loss["grad_logp"])
     assert rel_fro(np_(bw["grad_hidden"].float()), ref_bw["grad_hidden"]) <= TOL_GRAD
     assert rel_fro(np_(bw["grad_w"]), ref_bw["grad_w"]) <= TOL_GRAD
+
+
+def test_many_tiny_sequences():
+    """100,003 sequences of 0-5 tokens: dozens of sequences per persistent
+    CTA, and the last CTA's fixed-order sum over 100,003 per-sequence shares
+    (not a multiple of the 4-share vector loads)."""
+    lens = torch.randint(0, 6, (100_003,), generator=torch.Generator().manual_seed(13)).tolist()
+    compare(*make(lens, seed=14, mask_p=0.8), 0.2, 0.28)
