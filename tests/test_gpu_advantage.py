@@ -54,7 +54,8 @@ def test_degenerate_groups():
     check(*make(5, 3, 2), 1, 0.75, 0.5, 0.2, 1e-6)  # groups of one: advantage 0
 
 
-@pytest.mark.parametrize("T,G", [(40, 8), (96, 32), (48, 16), (34, 2), (60, 6), (36, 12), (1 << 16, 8)])
+@pytest.mark.parametrize("T,G", [(40, 8), (96, 32), (48, 16), (34, 2), (60, 6), (36, 12), (1 << 16, 8),
+                                 (24_008, 8), (24_000, 32), (24_001, 1)])  # many 512-row blocks, a partial last
 @pytest.mark.parametrize("K", [4, 3])  # 4 turns: vector row loads; 3: per-turn loads
 def test_group_sizes_and_batch_tails(T, G, K):
     check(*make(T, K, 3), G, 0.75, 0.5, 0.2, 1e-6)
