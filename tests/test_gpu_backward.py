@@ -112,8 +112,15 @@ def test_wide_tile_dz_long_hidden():
     check(*setup(4200, 8192, 300, seed=25))
 
 
+@pytest.mark.parametrize("N", [2048, 2304, 3000])
+def test_dz_tile_threshold(N):
+    """Kept-row counts around the switch of the dZ producer to 256-row tiles
+    (at 2304 rows), with the entropy term."""
+    check(*setup(N, 128, 900, seed=29))
+
+
 def test_wide_tile_dz_producer():
-    """>= 4096 kept rows: the dZ producer runs 256-row tiles (4500 rows =
+    """>= 2304 kept rows: the dZ producer runs 256-row tiles (4500 rows =
     17 blocks + 148), with the entropy term and temperature."""
     check(*setup(4500, 128, 1500, seed=14), inv_temp=1.0 / 0.9)
 

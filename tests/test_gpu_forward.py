@@ -53,7 +53,7 @@ def test_ragged_shapes(N, d, V):
 
 @pytest.mark.parametrize("inv_temp", [1.0, 1.0 / 0.9])
 def test_wide_tiles_ragged(inv_temp):
-    """>= 4096 rows: 256-row tiles with 8 epilogue warps (4500 rows = 17
+    """>= 2304 rows: 256-row tiles with 8 epilogue warps (4500 rows = 17
     blocks + 148), a vocabulary tail of 184 columns."""
     spec = workloads.spec_for(1, n_seqs=1, len_lo=4500, len_hi=4500, d=256, V=3000)
     run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
@@ -63,6 +63,14 @@ def test_million_entry_vocabulary():
     """V = 1,000,003 (3,907 tiles, a 3-column tail; the maximum 16 splits per
     row block) on 64 rows, d = 64."""
     spec = workloads.spec_for(1, n_seqs=1, len_lo=64, len_hi=64, d=64, V=1_000_003, seed=26)
+    run_and_compare(workloads.build(spec, "cpu"))
+
+
+@pytest.mark.parametrize("N", [2048, 2304, 3000])
+def test_wide_tile_threshold(N):
+    """The row counts around the switch to 256-row tiles (at 2304 rows):
+    2048 rows on 128-row tiles, exactly 9 wide row blocks, and 11 + 184."""
+    spec = workloads.spec_for(1, n_seqs=1, len_lo=N, len_hi=N, d=256, V=2000, seed=28)
     run_and_compare(workloads.build(spec, "cpu"))
 
 
