@@ -478,8 +478,10 @@ static int tile_group(int n_tiles, long long m_blocks, int conc, int rb) {
 }
 
 // K extent (in BK blocks) from which grad_hidden / grad_w use the wide
-// 256-row tile: the un-overlapped epilogue is then < 1 % of a unit.
-constexpr int kWideMinKBlocks = 256;
+// 256-row tile: measured on the 9B-class shapes, grad_w (K = kept rows) runs
+// ~2 % faster on it at K = 4,096 and 4-9 % faster at 6,144-12,288; its
+// un-overlapped epilogue stays small next to a K loop of 64+ blocks.
+constexpr int kWideMinKBlocks = 64;
 
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   Schedule sch;

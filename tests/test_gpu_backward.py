@@ -145,17 +145,30 @@ def test_row_chunks_across_the_wide_tile_threshold():
 
 
 def test_wide_tile_grad_hidden_long_vocabulary():
-    """K = V >= 256 k-blocks: grad_hidden runs 256-row tiles (600 rows =
+    """K = V >= 64 k-blocks: grad_hidden runs 256-row tiles (600 rows =
     2 blocks + 88, vocabulary tail of 33 columns)."""
     check(*setup(600, 256, 16481, seed=10))
 
 
 def test_wide_tile_grad_w_many_rows_with_accumulate():
-    """K = rows >= 256 k-blocks: grad_w runs 256-row vocabulary tiles
+    """K = rows >= 64 k-blocks: grad_w runs 256-row vocabulary tiles
     (V = 700 = 2 blocks + 188) over 16,500 rows, accumulating."""
     wl, g, ge = setup(16500, 128, 700, seed=11)
     base = torch.randn(700, 128, generator=torch.Generator().manual_seed(12))
     check(wl, g, ge, accumulate_base=base)
+
+
+@pytest.mark.parametrize("N", [4032, 4096, 4100])
+def test_grad_w_tile_threshold(N):
+    """grad_w's K (kept rows) around the switch to 256-row tiles at 64
+    k-blocks: 63 blocks, exactly 64, and 64 plus a 4-row tail block."""
+    check(*setup(N, 64, 500, seed=30))
+
+
+@pytest.mark.parametrize("V", [4032, 4097])
+def test_grad_hidden_tile_threshold(V):
+    """grad_hidden's K (the vocabulary) on both sides of 64 k-blocks."""
+    check(*setup(300, 128, V, seed=31))
 
 
 def test_wide_tile_with_short_device_count():
@@ -204,7 +217,7 @@ def test_row_keep_gate_equals_zeroed_upstream():
     assert rel_fro(np_(a["grad_w"]), ref["grad_w"]) <= TOL_GRAD
 
 
-@pytest.mark.parametrize("N", [300, 16500])  # grad_w on 128-row and on 256-row tiles
+@pytest.mark.parametrize("N", [300, 16500])  # grad_w on 128-row and on 256-row tiles (K >= 4096)
 def test_every_row_dropped(N):
     """row_keep all 0: no row has a gradient, so the device-side K of grad_w is
     0: grad_hidden and grad_w are zero, or grad_w keeps its value when
