@@ -250,6 +250,9 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.timeout_ns = wait_timeout_ns();
   a.pair = use_pair_engine() ? 1 : 0;
   a.wide = wide_rows(N) ? 1 : 0;
+  // Two column halves per sub-block when twice the split partials still fit
+  // the max_splits(V) slots per row that the workspace holds.
+  a.halves = (a.wide && 2 * a.splits <= max_splits(V)) ? 2 : 1;
   a.v_offset = v_offset;
   a.state = state;
   cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);

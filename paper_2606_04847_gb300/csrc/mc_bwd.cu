@@ -381,13 +381,13 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
                      cudaStream_t stream, int pair) {
   if (pair) return run_gemm_pair<Epi, A_MN, B_MN>(ta, tb, sch, ep, timeout_ns, status, stream);
   auto kern = gemm_persistent<Epi, A_MN, B_MN, MS>;
-  constexpr size_t smem = TileCfg<MS>::template smem_bytes<Epi>();
+  constexpr size_t smem = TileFor<Epi, MS>::template smem_bytes<Epi>();
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int units = sch.m_blocks * sch.splits;  // host upper bound; the kernel may find fewer
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(ta, tb, sch, ep, timeout_ns, status);
+  kern<<<grid, TileFor<Epi, MS>::THREADS, smem, stream>>>(ta, tb, sch, ep, timeout_ns, status);
   return launched();
 }
 

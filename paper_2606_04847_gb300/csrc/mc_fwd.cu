@@ -26,24 +26,35 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-struct FwdEpi {
-  struct Params {
-    const int32_t* targets;
-    long long N;
-    int V;
-    float scale2;  // inv_temperature * log2(e)
-    float inv_temp;
-    float* part;   // [3][splits][n_pad]
-    float* zy;     // [n_pad]
-    long long n_pad;
-    int splits;
-    int v_offset;  // global id of column 0 (a vocabulary shard), 0 for the full vocabulary
-  };
+struct FwdParams {
+  const int32_t* targets;
+  long long N;
+  int V;
+  float scale2;  // inv_temperature * log2(e)
+  float inv_temp;
+  float* part;   // [3][slots][n_pad]
+  float* zy;     // [n_pad]
+  long long n_pad;
+  int slots;     // partial states per row: vocabulary splits x column halves
+  int v_offset;  // global id of column 0 (a vocabulary shard), 0 for the full vocabulary
+};
+
+// H = 2 (256-row tiles only): two warp groups per 128-row sub-block, each
+// keeping its own online state over one half of every tile's 256 columns;
+// the two halves' states go to slots 2 split and 2 split + 1 and are merged
+// by the finalize kernel like any other split.
+template <int H>
+struct FwdEpiT {
+  using Params = FwdParams;
+  static constexpr int kColumnHalves = H;
+  static constexpr int kChunks = BN / 32 / H;  // 32-column chunks this warp reads per tile
 
   float m, s0, s1, t0, t1;
   int y;
+  int half = 0;
 
   __device__ __forceinline__ void setup(const Params&, long long, bool) {}
+  __device__ __forceinline__ void set_half(int h) { half = h; }
 
   __device__ __forceinline__ void begin(const Params& p, long long row, int, int) {
     m = -INFINITY;
@@ -91,7 +102,7 @@ struct FwdEpi {
   __device__ __forceinline__ void tile(const Params& p, long long row, int n_tile, uint32_t taddr) {
     const int v0 = n_tile * BN;
 #pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = half * kChunks; c < (half + 1) * kChunks; ++c) {
       float x[32];
       tmem_ld32(taddr + c * 32, x);
       const int vc = v0 + c * 32;
@@ -111,8 +122,8 @@ struct FwdEpi {
   }
 
   __device__ __forceinline__ void end(const Params& p, long long row, int, int split, bool ok) {
-    const long long plane = static_cast<long long>(p.splits) * p.n_pad;
-    const long long o = static_cast<long long>(split) * p.n_pad + row;
+    const long long plane = static_cast<long long>(p.slots) * p.n_pad;
+    const long long o = static_cast<long long>(split * H + half) * p.n_pad + row;
     p.part[o] = ok ? m : NAN;
     p.part[plane + o] = s0 + s1;
     p.part[2 * plane + o] = t0 + t1;
@@ -234,15 +245,16 @@ __global__ void merge_states_kernel(const float4* __restrict__ states, int P, lo
 
 }  // namespace
 
-template <int MS>
-cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdEpi::Params& ep, cudaStream_t stream) {
-  auto kern = gemm_persistent<FwdEpi, false, false, MS>;
-  constexpr size_t smem = TileCfg<MS>::template smem_bytes<FwdEpi>();
+template <int MS, int H>
+cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdParams& ep, cudaStream_t stream) {
+  using Epi = FwdEpiT<H>;
+  auto kern = gemm_persistent<Epi, false, false, MS>;
+  constexpr size_t smem = TileFor<Epi, MS>::template smem_bytes<Epi>();
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int units = sch.m_blocks * sch.splits;
   const int grid = units < a.grid ? units : a.grid;
-  kern<<<grid, TileCfg<MS>::THREADS, smem, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status);
+  kern<<<grid, TileFor<Epi, MS>::THREADS, smem, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status);
   return launched();
 }
 
@@ -264,7 +276,9 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
   sch.k_blocks = a.d / BK;
-  FwdEpi::Params ep;
+  const int halves = (a.wide && !a.pair && a.halves == 2) ? 2 : 1;
+  const int slots = a.splits * halves;
+  FwdParams ep;
   ep.targets = a.targets;
   ep.N = a.N;
   ep.V = a.V;
@@ -273,25 +287,27 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   ep.part = a.part;
   ep.zy = a.zy;
   ep.n_pad = a.n_pad;
-  ep.splits = a.splits;
+  ep.slots = slots;
   ep.v_offset = a.v_offset;
   if (a.pair) {
-    e = run_gemm_pair<FwdEpi, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
+    e = run_gemm_pair<FwdEpiT<1>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
+  } else if (a.wide && halves == 2) {
+    e = run_forward_gemm<2, 2>(a, sch, ep, stream);
   } else if (a.wide) {
-    e = run_forward_gemm<2>(a, sch, ep, stream);
+    e = run_forward_gemm<2, 1>(a, sch, ep, stream);
   } else {
-    e = run_forward_gemm<1>(a, sch, ep, stream);
+    e = run_forward_gemm<1, 1>(a, sch, ep, stream);
   }
   if (e != cudaSuccess) return e;
   const int threads = 256;
   const long long blocks = (a.N + threads - 1) / threads;
   if (a.state != nullptr)
     fwd_state_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-        a.targets, a.N, a.V, a.v_offset, a.splits, a.n_pad, a.part, a.zy, reinterpret_cast<float4*>(a.state),
+        a.targets, a.N, a.V, a.v_offset, slots, a.n_pad, a.part, a.zy, reinterpret_cast<float4*>(a.state),
         a.ws_status, a.dev_status);
   else
     fwd_finalize<<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-        a.targets, a.N, a.V, a.splits, a.n_pad, a.part, a.zy, a.logp, a.entropy, a.lse, a.ws_status,
+        a.targets, a.N, a.V, slots, a.n_pad, a.part, a.zy, a.logp, a.entropy, a.lse, a.ws_status,
         a.dev_status);
   return launched();
 }

@@ -6,16 +6,17 @@
 // forward turns it into an online log-sum-exp / entropy update, the backward
 // into dZ, the backward GEMMs into plain stores.
 //
-// CTA = 2 + 4 * MS warps, one CTA per SM (the SMEM ring takes 192 KB, plus
+// CTA = 2 + 4 * MS * H warps, one CTA per SM (the SMEM ring takes 192 KB, plus
 // the epilogue's own staging buffers when it asks for them):
 //   warp 0        TMA producer: loads A/B k-blocks (BK = 64) into the ring
 //                 (4 x 48 KB stages; 3 x 64 KB with MS = 2)
 //   warp 1        TMEM allocator + MMA issuer (one thread): 4 x MS
 //                 tcgen05.mma (M=128, N=256, K=16) per k-block into TMEM
 //                 (2 x 256 fp32 columns = all 512 columns)
-//   warps 2..     epilogue (4 warps per 128-row sub-block): warp w reads TMEM
-//                 lanes 32*(w%4)..+31 of its sub-block, one output row per
-//                 thread, 32 columns per tcgen05.ld
+//   warps 2..     epilogue (4 warps per 128-row sub-block, or per sub-block
+//                 and column half when the epilogue asks for H = 2 halves):
+//                 warp w reads TMEM lanes 32*(w%4)..+31 of its sub-block, one
+//                 output row per thread, 32 columns per tcgen05.ld
 // With MS = 1 the two 256-column accumulators let the epilogue of tile j
 // overlap the MMAs of tile j+1; with MS = 2 they hold the two 128-row halves
 // of one 256 x 256 tile (see TileCfg). Barriers: full[s]/empty[s] per ring
@@ -87,6 +88,20 @@ struct EpiStage<E, std::void_t<decltype(E::kStageBytes)>> {
 };
 constexpr size_t kEpiStageOffset = (size_t(NUM_STAGES) * STAGE_BYTES + sizeof(GemmShared) + 1023) / 1024 * 1024;
 
+// Epilogues may also ask, through `static constexpr int kColumnHalves = 2`,
+// for two warp groups per 128-row sub-block of a 256-row tile, each draining
+// half of the tile's 256 columns (16 epilogue warps: twice the warps hiding
+// TMEM-load and arithmetic latency while the MMAs wait for the drain). The
+// engine then calls `epi.set_half(h)` once, h = the warp's column half.
+template <class E, class = void>
+struct EpiColumnHalves {
+  static constexpr int value = 1;
+};
+template <class E>
+struct EpiColumnHalves<E, std::void_t<decltype(E::kColumnHalves)>> {
+  static constexpr int value = E::kColumnHalves;
+};
+
 enum DynMode : int { DYN_NONE = 0, DYN_ROWS = 1, DYN_K = 2 };
 
 struct Schedule {
@@ -151,14 +166,16 @@ struct Schedule {
 // fewer from L2, and its ring covers longer operand latency; the epilogue no
 // longer overlaps the MMAs, which costs a GEMM little when its K loop is long
 // or its epilogue short. Unit row blocks are then 256 rows.
-template <int MS>
+template <int MS, int H = 1>
 struct TileCfg {
   static_assert(MS == 1 || MS == 2, "one or two 128-row sub-blocks");
+  static_assert(H == 1 || (H == 2 && MS == 2), "column halves only with 256-row tiles");
   static constexpr int TBM = BM * MS;
   static constexpr int STAGES = MS == 1 ? NUM_STAGES : 3;
   static constexpr int SBYTES = MS * A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr int SLOTS = NUM_ACC / MS;  // tiles in flight in TMEM
-  static constexpr int EPI_WARPS = NUM_EPI_WARPS * MS;  // 4 per 128-row sub-block
+  static constexpr int HALVES = H;            // warp groups per sub-block (column halves)
+  static constexpr int EPI_WARPS = NUM_EPI_WARPS * MS * H;  // 4 per 128-row sub-block and column half
   static constexpr int THREADS = 32 * (EPI_WARP_BEGIN + EPI_WARPS);
   // Dynamic shared memory of the kernel running epilogue E.
   template <class E>
@@ -170,13 +187,19 @@ struct TileCfg {
   static_assert(STAGES <= NUM_STAGES && SLOTS >= 1, "barrier arrays are sized for the narrow tile");
 };
 
+// The tile configuration a kernel with epilogue E and MS sub-blocks runs:
+// E's column halves apply to 256-row tiles only.
+template <class E, int MS>
+using TileFor = TileCfg<MS, (MS == 2 ? EpiColumnHalves<E>::value : 1)>;
+
 template <class Epi, bool A_MN, bool B_MN, int MS = 1>
-__global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
+__global__ void __launch_bounds__(TileFor<Epi, MS>::THREADS, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const Schedule sch_in, const __grid_constant__ typename Epi::Params ep,
                     const uint64_t timeout_ns, int32_t* dev_status) {
-  using C = TileCfg<MS>;
+  using C = TileFor<Epi, MS>;
   static_assert(C::template smem_bytes<Epi>() <= 227 * 1024, "shared memory of one CTA exceeded");
+  static_assert(C::HALVES == 1 || EpiStage<Epi>::bytes == 0, "column halves are for epilogues without staging");
   Schedule sch = sch_in;
   long long rows_eff = -1;
   bool k_nonempty = true;
@@ -325,9 +348,12 @@ __global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    // Warps 2.. in groups of four, group j draining row sub-block j; within a
-    // group, warp w may access TMEM lane quadrant w % 4 only.
-    const int sub = (warp - EPI_WARP_BEGIN) / NUM_EPI_WARPS;
+    // Warps 2.. in groups of four, group g draining row sub-block g % MS
+    // (and, with two column halves, columns [128 h, 128 h + 128) of it,
+    // h = g / MS); within a group, warp w may access TMEM lane quadrant w % 4
+    // only.
+    const int group = (warp - EPI_WARP_BEGIN) / NUM_EPI_WARPS;
+    const int sub = group % MS;
     const int quad = warp & 3;
     const int row_in_tile = sub * BM + quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
@@ -336,6 +362,7 @@ __global__ void __launch_bounds__(TileCfg<MS>::THREADS, 1)
     epi.setup(ep, rows_eff, k_nonempty);
     if constexpr (EpiStage<Epi>::bytes > 0)
       epi.stage(smem + kEpiStageOffset + (warp - EPI_WARP_BEGIN) * EpiStage<Epi>::bytes);
+    if constexpr (C::HALVES > 1) epi.set_half(group / MS);
     bool ok = true;
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       int mb, split, t0, t1;

@@ -30,7 +30,7 @@ struct FwdArgs {
   float inv_temperature;
   int splits;
   long long n_pad;
-  float* part;            // workspace: [3][splits][n_pad]
+  float* part;            // workspace: [3][splits * halves][n_pad]
   float* zy;              // workspace: [n_pad]
   int32_t* ws_status;     // workspace: internal status word (zeroed by the caller)
   float* logp;
@@ -41,6 +41,8 @@ struct FwdArgs {
   uint64_t timeout_ns;
   int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
   int wide;               // one-CTA engine only: 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
+  int halves;             // 256-row tiles: 2 = two epilogue warp groups per sub-block, one per
+                          // column half, each with its own partial slot (needs 2 * splits <= 16)
   int v_offset;           // global vocabulary id of W's row 0 (shards); 0 otherwise
   float* state;           // non-null: write the slice state [N, 4] instead of logp/entropy/lse
 };
