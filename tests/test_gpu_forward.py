@@ -53,7 +53,8 @@ def test_ragged_shapes(N, d, V):
 
 @pytest.mark.parametrize("inv_temp", [1.0, 1.0 / 0.9])
 def test_wide_tiles_ragged(inv_temp):
-    """>= 2304 rows: 256-row tiles with 8 epilogue warps (4500 rows = 17
+    """>= 2304 rows: 256-row tiles with 16 epilogue warps over two column
+    halves when twice the splits fit the workspace, else 8 (4500 rows = 17
     blocks + 148), a vocabulary tail of 184 columns."""
     spec = workloads.spec_for(1, n_seqs=1, len_lo=4500, len_hi=4500, d=256, V=3000)
     run_and_compare(workloads.build(spec, "cpu"), inv_temp=inv_temp)
