@@ -161,7 +161,8 @@ struct Schedule {
 // two tiles in flight in TMEM (the epilogue of one overlaps the MMAs of the
 // next). MS = 2 ("wide"): 256 x 256 tiles computed as two M = 128 MMAs that
 // share each B stage, 3 x 64 KB stages, both TMEM accumulators on the one
-// tile in flight, and 8 epilogue warps that drain the two halves at once. A
+// tile in flight, and 8 epilogue warps that drain the two halves at once (16
+// when the epilogue asks for H = 2 column halves). A
 // wide tile streams ~29 % fewer operand bytes per output from HBM and a third
 // fewer from L2, and its ring covers longer operand latency; the epilogue no
 // longer overlaps the MMAs, which costs a GEMM little when its K loop is long
