@@ -64,17 +64,9 @@ mc_status device_info(int* sms) {
   return MC_OK;
 }
 
-uint64_t wait_timeout_ns() {
-  static const uint64_t t = [] {
-    const char* s = std::getenv("MC_WAIT_TIMEOUT_NS");
-    if (s != nullptr) {
-      const unsigned long long v = std::strtoull(s, nullptr, 10);
-      if (v >= 1000000ull && v <= 60000000000ull) return static_cast<uint64_t>(v);
-    }
-    return static_cast<uint64_t>(4000000000ull);  // 4 s: far above any healthy wait
-  }();
-  return t;
-}
+// Limit of every bounded pipeline wait: far above any healthy wait (the
+// longest, an MMA issuer waiting for one operand stage, takes microseconds).
+constexpr uint64_t kWaitTimeoutNs = 4000000000ull;  // 4 s
 
 // ---- TMA descriptors
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -229,7 +221,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   mc::FwdArgs a;
   if ((st = make_tmap(&a.tm_hidden, hidden, d, N, d, kBM)) != MC_OK) return st;
-  if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, b_box_rows())) != MC_OK) return st;
+  if ((st = make_tmap(&a.tm_w, w_vocab, d, V, d, kBN)) != MC_OK) return st;
   const long long m_blocks = ceil_div(N, row_block(N));
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
   a.targets = targets;
@@ -247,8 +239,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.lse = lse;
   a.dev_status = dev_status;
   a.grid = sms;
-  a.timeout_ns = wait_timeout_ns();
-  a.pair = use_pair_engine() ? 1 : 0;
+  a.timeout_ns = kWaitTimeoutNs;
   a.wide = wide_rows(N) ? 1 : 0;
   // Two column halves per sub-block when twice the split partials still fit
   // the max_splits(V) slots per row that the workspace holds.
@@ -365,7 +356,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
   if ((e = cudaMemsetAsync(grad_hidden, 0, size_t(N) * size_t(d) * 2, s)) != cudaSuccess)
     return cuda_fail(e, "cudaMemsetAsync");
 
-  const uint64_t tmo = wait_timeout_ns();
+  const uint64_t tmo = kWaitTimeoutNs;
   mc::SelectArgs sa;
   sa.hidden = hidden;
   sa.row_keep = row_keep;
@@ -387,7 +378,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
   if ((e = mc::launch_select_gather(sa, s)) != cudaSuccess) return cuda_fail(e, "row selection launch");
 
   CUtensorMap tm_w_k, tm_w_mn;
-  if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, b_box_rows())) != MC_OK) return st;
+  if ((st = make_tmap(&tm_w_k, w_vocab, d, V, d, kBN)) != MC_OK) return st;
   if ((st = make_tmap(&tm_w_mn, w_vocab, d, V, d, 64)) != MC_OK) return st;
   const int n_tiles = static_cast<int>(ceil_div(V, kBN));
 
@@ -418,7 +409,6 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.ws_status = ws_status;
     za.grid = sms;
     za.timeout_ns = tmo;
-    za.pair = use_pair_engine() ? 1 : 0;
     za.wide = wide_rows(rows) ? 1 : 0;
     if ((e = mc::launch_dz(za, s)) != cudaSuccess) return cuda_fail(e, "dZ launch");
 
@@ -435,7 +425,6 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     ha.ws_status = ws_status;
     ha.grid = sms;
     ha.timeout_ns = tmo;
-    ha.pair = use_pair_engine() ? 1 : 0;
     if ((e = mc::launch_dh(ha, s)) != cudaSuccess) return cuda_fail(e, "dH launch");
 
     mc::DwArgs wa;
@@ -451,7 +440,6 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     wa.ws_status = ws_status;
     wa.grid = sms;
     wa.timeout_ns = tmo;
-    wa.pair = use_pair_engine() ? 1 : 0;
     if ((e = mc::launch_dw(wa, s)) != cudaSuccess) return cuda_fail(e, "dW launch");
   }
   if ((e = mc::launch_status_merge(ws_status, dev_status, s)) != cudaSuccess) return cuda_fail(e, "status launch");

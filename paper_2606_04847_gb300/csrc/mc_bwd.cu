@@ -22,7 +22,6 @@
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
-#include "mc_gemm2.cuh"
 #include "mc_internal.h"
 
 namespace mc {
@@ -32,6 +31,7 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kSelectThreads = 1024;
+constexpr int kHcRowPad = 2 * BM;  // gathered rows are zero-padded to whole 256-row blocks
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -136,11 +136,11 @@ __global__ void __launch_bounds__(kSelectThreads) select_write_kernel(
 }
 
 // Hc[j] = H[idx[j]] for j < count, zero rows up to the next multiple of 256
-// (a whole row block of either engine).
+// (a whole row block of either tile height).
 __global__ void gather_rows_kernel(const uint4* __restrict__ H, int row_vec, const int32_t* __restrict__ idx,
                                    const int32_t* __restrict__ count, uint4* __restrict__ Hc) {
   const long long cnt = *count;
-  const long long lim = (cnt + PAIR_BM - 1) / PAIR_BM * PAIR_BM;
+  const long long lim = (cnt + kHcRowPad - 1) / kHcRowPad * kHcRowPad;
   for (long long j = blockIdx.x; j < lim; j += gridDim.x) {
     uint4* dst = Hc + j * row_vec;
     if (j < cnt) {
@@ -166,8 +166,6 @@ struct DzParams {
   int V;
   float scale2;
   float inv_temp;
-  __nv_bfloat16* dz;
-  long long ld;
 };
 
 // kEntropy = false when there is no entropy gradient (gH == 0 for every row):
@@ -176,13 +174,12 @@ template <bool kEntropy>
 struct DzEpi {
   using Params = DzParams;
 
-  // Staged stores (one-CTA engine): each epilogue warp writes its 32 rows x
-  // 32 columns of bf16 into one of two 2 KB shared-memory buffers in the
-  // 64-byte swizzle (row r's 16-byte piece q at position q ^ ((r >> 1) & 3),
-  // conflict-free), and one lane stores the box with TMA: whole lines reach
-  // L2 instead of 32 scattered 16-byte pieces per warp store instruction.
-  // The tensor map's extent clips rows past the chunk and columns past V.
-  // Without a buffer (the CTA-pair engine) each thread stores its own row.
+  // Staged stores: each epilogue warp writes its 32 rows x 32 columns of
+  // bf16 into one of two 2 KB shared-memory buffers in the 64-byte swizzle
+  // (row r's 16-byte piece q at position q ^ ((r >> 1) & 3), conflict-free),
+  // and one lane stores the box with TMA: whole lines reach L2 instead of 32
+  // scattered 16-byte pieces per warp store instruction. The tensor map's
+  // extent clips rows past the chunk and columns past V.
   static constexpr int kStageBytes = 4096;
 
   long long rows_lim;
@@ -194,7 +191,6 @@ struct DzEpi {
 
   __device__ __forceinline__ void setup(const Params& p, long long rows_eff, bool) {
     rows_lim = rows_eff >= 0 ? rows_eff : p.rows;
-    sbuf = nullptr;
     nstore = 0;
   }
   __device__ __forceinline__ void stage(uint8_t* buf) { sbuf = buf; }
@@ -227,7 +223,6 @@ struct DzEpi {
       tmem_ld32(taddr + c * 32, x);
       const int vc = v0 + c * 32;
       if (vc >= p.V) continue;  // the same for the whole warp
-      if (sbuf == nullptr && row >= p.rows) continue;
       uint32_t w[16];
       if (valid) {
         const float nl = -lse2;
@@ -261,37 +256,22 @@ struct DzEpi {
 #pragma unroll
         for (int i = 0; i < 16; ++i) w[i] = 0u;
       }
-      if (sbuf != nullptr) {
-        const int lane = threadIdx.x & 31;
-        if (row - lane >= p.rows) continue;  // the warp's rows all lie past the chunk: nothing to store
-        uint8_t* buf = sbuf + (nstore & 1u) * 2048u;
-        if (lane == 0) bulk_wait_group_read<1>();  // the store that last used this buffer has read it
-        __syncwarp();
-        uint4* r4 = reinterpret_cast<uint4*>(buf + lane * 64);
-        const int sw = (lane >> 1) & 3;
+      const int lane = threadIdx.x & 31;
+      if (row - lane >= p.rows) continue;  // the warp's rows all lie past the chunk: nothing to store
+      uint8_t* buf = sbuf + (nstore & 1u) * 2048u;
+      if (lane == 0) bulk_wait_group_read<1>();  // the store that last used this buffer has read it
+      __syncwarp();
+      uint4* r4 = reinterpret_cast<uint4*>(buf + lane * 64);
+      const int sw = (lane >> 1) & 3;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) r4[q ^ sw] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-        fence_proxy_async_shared();
-        __syncwarp();
-        if (lane == 0) {
-          tma_store_2d(&p.tm_st, buf, vc, static_cast<int32_t>(row - lane));
-          bulk_commit_group();
-        }
-        ++nstore;
-        continue;
+      for (int q = 0; q < 4; ++q) r4[q ^ sw] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+      fence_proxy_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(&p.tm_st, buf, vc, static_cast<int32_t>(row - lane));
+        bulk_commit_group();
       }
-      __nv_bfloat16* dst = p.dz + row * p.ld + vc;
-      if (vc + 32 <= p.V) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) __stcs(d4 + q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]));
-      } else {
-        const int n = p.V - vc;
-        uint16_t* d16 = reinterpret_cast<uint16_t*>(dst);
-#pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (i < n) d16[i] = static_cast<uint16_t>((i & 1) ? (w[i / 2] >> 16) : (w[i / 2] & 0xFFFFu));
-      }
+      ++nstore;
     }
   }
 
@@ -378,8 +358,7 @@ struct StoreF32Epi {
 template <class Epi, bool A_MN, bool B_MN, int MS = 1>
 cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedule& sch,
                      const typename Epi::Params& ep, int grid_cap, uint64_t timeout_ns, int32_t* status,
-                     cudaStream_t stream, int pair) {
-  if (pair) return run_gemm_pair<Epi, A_MN, B_MN>(ta, tb, sch, ep, timeout_ns, status, stream);
+                     cudaStream_t stream) {
   auto kern = gemm_persistent<Epi, A_MN, B_MN, MS>;
   constexpr size_t smem = TileFor<Epi, MS>::template smem_bytes<Epi>();
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -422,7 +401,7 @@ cudaError_t launch_select_gather(const SelectArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   Schedule sch;
-  const int rb = a.pair ? PAIR_BM : (a.wide ? 2 * BM : BM);
+  const int rb = a.wide ? 2 * BM : BM;
   sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
@@ -442,21 +421,19 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   ep.V = a.V;
   ep.scale2 = a.inv_temperature * kLog2e;
   ep.inv_temp = a.inv_temperature;
-  ep.dz = static_cast<__nv_bfloat16*>(a.dz);
-  ep.ld = a.ld;
   ep.tm_st = a.tm_dz_st;
-  if (a.wide && !a.pair) {
+  if (a.wide) {
     if (a.grad_entropy != nullptr)
       return run_gemm<DzEpi<true>, false, false, 2>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns,
-                                                    a.ws_status, stream, 0);
+                                                    a.ws_status, stream);
     return run_gemm<DzEpi<false>, false, false, 2>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns,
-                                                   a.ws_status, stream, 0);
+                                                   a.ws_status, stream);
   }
   if (a.grad_entropy != nullptr)
     return run_gemm<DzEpi<true>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                               stream, a.pair);
+                                               stream);
   return run_gemm<DzEpi<false>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                              stream, a.pair);
+                                              stream);
 }
 
 // Tiles per group for a one-tile-per-unit long-K GEMM whose waves hold `conc`
@@ -486,12 +463,12 @@ constexpr int kWideMinKBlocks = 64;
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   Schedule sch;
   sch.k_blocks = (a.V + BK - 1) / BK;
-  const bool wide = !a.pair && sch.k_blocks >= kWideMinKBlocks;
-  const int rb = a.pair ? PAIR_BM : (wide ? 2 * BM : BM);
+  const bool wide = sch.k_blocks >= kWideMinKBlocks;
+  const int rb = wide ? 2 * BM : BM;
   sch.m_blocks = static_cast<int>((a.rows + rb - 1) / rb);
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;  // one output tile per unit
-  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
+  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
@@ -504,20 +481,20 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   ep.cols = a.d;
   if (wide)
     return run_gemm<StoreBf16Epi, false, true, 2>(a.tm_dz, a.tm_w_mn, sch, ep, a.grid, a.timeout_ns,
-                                                  a.ws_status, stream, 0);
+                                                  a.ws_status, stream);
   return run_gemm<StoreBf16Epi, false, true>(a.tm_dz, a.tm_w_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                             stream, a.pair);
+                                             stream);
 }
 
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   Schedule sch;
   sch.k_blocks = static_cast<int>((a.rows + BK - 1) / BK);  // host bound; the kernel reads the count
-  const bool wide = !a.pair && sch.k_blocks >= kWideMinKBlocks;
-  const int rb = a.pair ? PAIR_BM : (wide ? 2 * BM : BM);
+  const bool wide = sch.k_blocks >= kWideMinKBlocks;
+  const int rb = wide ? 2 * BM : BM;
   sch.m_blocks = (a.V + rb - 1) / rb;
   sch.n_tiles = (a.d + BN - 1) / BN;
   sch.splits = sch.n_tiles;
-  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.pair ? a.grid / 2 : a.grid, rb);
+  sch.n_group = tile_group(sch.n_tiles, sch.m_blocks, a.grid, rb);
   sch.dyn_count = a.count;
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
@@ -530,9 +507,9 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   ep.accumulate = a.accumulate;
   if (wide)
     return run_gemm<StoreF32Epi, true, true, 2>(a.tm_dz_mn, a.tm_h_mn, sch, ep, a.grid, a.timeout_ns,
-                                                a.ws_status, stream, 0);
+                                                a.ws_status, stream);
   return run_gemm<StoreF32Epi, true, true>(a.tm_dz_mn, a.tm_h_mn, sch, ep, a.grid, a.timeout_ns, a.ws_status,
-                                           stream, a.pair);
+                                           stream);
 }
 
 cudaError_t launch_status_merge(const int32_t* ws_status, int32_t* dev_status, cudaStream_t stream) {

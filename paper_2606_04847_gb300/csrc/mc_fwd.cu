@@ -16,7 +16,6 @@
 #include <cuda_bf16.h>
 
 #include "mc_gemm.cuh"
-#include "mc_gemm2.cuh"
 #include "mc_internal.h"
 
 namespace mc {
@@ -271,12 +270,12 @@ cudaError_t launch_merge_states(const float* states, int P, long long N, float* 
 cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   cudaError_t e;
   Schedule sch;
-  const int row_block = a.pair ? PAIR_BM : (a.wide ? 2 * BM : BM);
+  const int row_block = a.wide ? 2 * BM : BM;
   sch.m_blocks = static_cast<int>((a.N + row_block - 1) / row_block);
   sch.n_tiles = (a.V + BN - 1) / BN;
   sch.splits = a.splits;
   sch.k_blocks = a.d / BK;
-  const int halves = (a.wide && !a.pair && a.halves == 2) ? 2 : 1;
+  const int halves = (a.wide && a.halves == 2) ? 2 : 1;
   const int slots = a.splits * halves;
   FwdParams ep;
   ep.targets = a.targets;
@@ -289,9 +288,7 @@ cudaError_t launch_forward(const FwdArgs& a, cudaStream_t stream) {
   ep.n_pad = a.n_pad;
   ep.slots = slots;
   ep.v_offset = a.v_offset;
-  if (a.pair) {
-    e = run_gemm_pair<FwdEpiT<1>, false, false>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status, stream);
-  } else if (a.wide && halves == 2) {
+  if (a.wide && halves == 2) {
     e = run_forward_gemm<2, 2>(a, sch, ep, stream);
   } else if (a.wide) {
     e = run_forward_gemm<2, 1>(a, sch, ep, stream);

@@ -39,8 +39,7 @@ struct FwdArgs {
   int32_t* dev_status;
   int grid;
   uint64_t timeout_ns;
-  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
-  int wide;               // one-CTA engine only: 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
+  int wide;               // 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
   int halves;             // 256-row tiles: 2 = two epilogue warp groups per sub-block, one per
                           // column half, each with its own partial slot (needs 2 * splits <= 16)
   int v_offset;           // global vocabulary id of W's row 0 (shards); 0 otherwise
@@ -90,8 +89,7 @@ struct DzArgs {
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
-  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
-  int wide;               // one-CTA engine only: 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
+  int wide;               // 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
 };
 cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream);
 
@@ -107,7 +105,6 @@ struct DhArgs {           // grad_hidden[idx[j], :] = (dZ . W)[j, :]
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
-  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream);
 
@@ -123,7 +120,6 @@ struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . Hc[rows, d]
   int32_t* ws_status;
   int grid;
   uint64_t timeout_ns;
-  int pair;               // 1: CTA-pair engine (cta_group::2), 0: one-CTA engine
 };
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream);
 

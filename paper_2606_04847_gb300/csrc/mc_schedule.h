@@ -1,51 +1,33 @@
 // mc_schedule.h — the launch-shaping policy of the C-ABI layer (host code,
-// included by mc_api.cu only): which GEMM engine runs, the row-block height
-// of a projection launch, and how many vocabulary splits its row blocks get.
+// included by mc_api.cu only): the row-block height of a projection launch, and how many vocabulary splits its row blocks get.
 // These choices decide how often W is streamed from HBM and how busy the SMs
 // are; the kernels themselves live in mc_gemm.cuh / mc_fwd.cu / mc_bwd.cu.
 #pragma once
 
 #include <cmath>
-#include <cstdlib>
-#include <cstring>
 
 namespace mc {
 namespace sched {
 
 constexpr int kBM = 128;       // rows one CTA owns in a tile (TMA box height for A)
 constexpr int kBN = 256;       // vocabulary / output columns per tile
-constexpr int kRowPad = 256;   // row padding of workspaces: one row block of either engine
+constexpr int kRowPad = 256;   // row padding of workspaces: one row block of either tile height
 constexpr int kMaxSplits = 16;
 
 inline long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 
-// The one-CTA engine unless MC_ENGINE=pair selects the CTA-pair engine
-// (tcgen05 cta_group::2). Both give the same results; under the GB300's power
-// cap the one-CTA engine sustains a ~10 % higher SM clock, and its 9B-class
-// step ran ~4 % faster before its 256-row tiles and ~12 % faster with them,
-// so it is the default.
-inline bool use_pair_engine() {
-  static const bool pair = [] {
-    const char* s = std::getenv("MC_ENGINE");
-    return s != nullptr && std::strcmp(s, "pair") == 0;
-  }();
-  return pair;
-}
-
-// Projection launches (forward, dZ) of the one-CTA engine with at least this
+// Projection launches (forward, dZ) with at least this
 // many rows use 256-row tiles (TileCfg<2>: a third less operand traffic per
 // FLOP, 8 epilogue warps); fewer rows keep 128-row tiles so that small
 // launches still spread over the SMs. Measured on the 9B-class shapes: the
 // 256-row forward is 7-10 % faster from 2,304 rows up and 1 % slower at 2,048.
 constexpr long long kWideMinRows = 2304;
-inline bool wide_rows(long long rows) { return !use_pair_engine() && rows >= kWideMinRows; }
+inline bool wide_rows(long long rows) { return rows >= kWideMinRows; }
 
-// Rows per scheduled row block of a projection launch over `rows` rows, TMA
-// box height of K-major B, and how many units run at once, for the selected
-// engine.
-inline int row_block(long long rows) { return (use_pair_engine() || wide_rows(rows)) ? 256 : kBM; }
-inline int b_box_rows() { return use_pair_engine() ? 128 : kBN; }
-inline int concurrent_units(int sms) { return use_pair_engine() ? sms / 2 : sms; }
+// Rows per scheduled row block of a projection launch over `rows` rows; one
+// unit runs per SM at a time.
+inline int row_block(long long rows) { return wide_rows(rows) ? 256 : kBM; }
+inline int concurrent_units(int sms) { return sms; }
 
 // Vocabulary tile ranges per row block. A wave of `conc` concurrent units
 // streams W once and keeps its conc / s row blocks of hidden rows in L2, so
