@@ -1,7 +1,7 @@
 """GPU backward (mc_token_logprobs_bwd) vs the fp64 oracle's closed form.
 
-Relative Frobenius error of grad_hidden and grad_w <= 1e-2, plus a per-row
-check on rows with a nonzero upstream gradient, over ragged shapes, several
+Relative Frobenius error of grad_hidden and grad_w <= 1e-2, and the same
+bound on every grad_hidden row with a nonzero upstream gradient, over ragged shapes, several
 row chunks (small workspace), accumulation into grad_w, the entropy term,
 temperature and rows skipped by the keep-mask (zero upstream gradient).
 """
@@ -48,10 +48,10 @@ def check(wl, grad_logp, grad_ent, inv_temp=1.0, rows_per_chunk=None, accumulate
     nzmask = (grad_logp != 0).numpy()
     if grad_ent is not None:
         nzmask |= (grad_ent != 0).numpy()
-    nz = np.nonzero(nzmask)[0]
-    for r in nz[:: max(1, len(nz) // 16)]:
+    # Every row with a nonzero upstream gradient, at the stated bound.
+    for r in np.nonzero(nzmask)[0]:
         er = rel_fro(gh[r], ref["grad_hidden"][r])
-        assert er <= 2 * TOL_GRAD, f"row {r}: rel err {er:.3e}"
+        assert er <= TOL_GRAD, f"row {r}: rel err {er:.3e}"
     return out, ref
 
 

@@ -155,7 +155,7 @@ def test_backward_full_size_9b():
             assert not got[i].any(), f"dropped row {r} has a gradient"
         else:
             e = rel_fro(got[i], ref["grad_hidden"][i])
-            assert e <= 2 * TOL_GRAD, f"row {r}: rel err {e:.3e}"
+            assert e <= TOL_GRAD, f"row {r}: rel err {e:.3e}"
 
     # <grad_hidden, H> = <grad_w, W>, in fp64 on the GPU.
     # Tolerance: 1e-2 relative plus the bf16 rounding of grad_hidden itself
