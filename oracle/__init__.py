@@ -25,7 +25,7 @@ force, closed forms, invariants, library routines, finite differences and the
 paper's worked example); none is "parity unpinned".
 """
 
-from .logprobs import logits, logprob_state, token_logprobs, token_logprobs_bwd  # noqa: F401
+from .logprobs import logprob_state, token_logprobs, token_logprobs_bwd, token_logprobs_bwd_rows  # noqa: F401
 from .filter import seq_ratio_filter  # noqa: F401
 from .grpo import grpo_masked_loss  # noqa: F401
 from .advantage import group_advantage, prime_echo_reward  # noqa: F401

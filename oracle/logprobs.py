@@ -46,7 +46,7 @@ from __future__ import annotations
 
 import numpy as np
 
-__all__ = ["as_f64", "logits", "token_logprobs", "token_logprobs_bwd"]
+__all__ = ["as_f64", "logprob_state", "token_logprobs", "token_logprobs_bwd", "token_logprobs_bwd_rows"]
 
 
 def as_f64(x) -> np.ndarray:
@@ -68,13 +68,6 @@ def as_i64(x) -> np.ndarray:
             x = x.cpu()
         return x.to(dtype=__import__("torch").int64).numpy()
     return np.asarray(x, dtype=np.int64)
-
-
-def logits(hidden, w_vocab, inv_temperature: float = 1.0) -> np.ndarray:
-    """z = (H W^T) * inv_temperature in float64 (the LM-head projection)."""
-    h = as_f64(hidden)
-    w = as_f64(w_vocab)
-    return (h @ w.T) * float(inv_temperature)
 
 
 def _row_stats(z: np.ndarray, y: np.ndarray):
@@ -160,6 +153,16 @@ def token_logprobs_bwd(hidden, w_vocab, targets, grad_logp, grad_entropy=None,
     g = as_f64(grad_logp)
     gh = np.zeros_like(g) if grad_entropy is None else as_f64(grad_entropy)
     z = (h @ w.T) * float(inv_temperature)
+    dz = _dz_rows(z, y, g, gh, inv_temperature)
+    out = {"grad_hidden": dz @ w, "grad_w": dz.T @ h}
+    if return_dz:
+        out["dz"] = dz
+    return out
+
+
+def _dz_rows(z: np.ndarray, y: np.ndarray, g: np.ndarray, gh: np.ndarray, inv_temperature: float) -> np.ndarray:
+    """dZ of a block of rows from their logits z [R, V] (module docstring):
+    the two-pass log-softmax, the entropy, then the closed form."""
     m = z.max(axis=1)
     lse = m + np.log(np.exp(z - m[:, None]).sum(axis=1))
     logp_all = z - lse[:, None]
@@ -167,9 +170,39 @@ def token_logprobs_bwd(hidden, w_vocab, targets, grad_logp, grad_entropy=None,
     ent = -(p * logp_all).sum(axis=1)
     onehot = np.zeros_like(z)
     onehot[np.arange(z.shape[0]), y] = 1.0
-    dz = float(inv_temperature) * (g[:, None] * (onehot - p)
-                                   - gh[:, None] * p * (logp_all + ent[:, None]))
-    out = {"grad_hidden": dz @ w, "grad_w": dz.T @ h}
-    if return_dz:
-        out["dz"] = dz
-    return out
+    return float(inv_temperature) * (g[:, None] * (onehot - p) - gh[:, None] * p * (logp_all + ent[:, None]))
+
+
+def token_logprobs_bwd_rows(hidden, w_vocab, targets, grad_logp, grad_entropy=None,
+                            inv_temperature: float = 1.0, vocab_rows=None, rows_per_block: int = 256):
+    """The closed-form gradients of ``token_logprobs_bwd`` for problems too
+    large to form Z whole: every row of grad_hidden, and grad_w at the
+    vocabulary rows ``vocab_rows`` only (all rows when None).
+
+    Rows t are independent up to dZ, so dZ is formed one block of rows at a
+    time, each row over the full vocabulary (nothing in a row's log-softmax,
+    entropy or dZ is blocked), and grad_hidden = dZ W per block. The columns
+    vocab_rows of dZ are kept for all rows, and grad_w[vocab_rows] =
+    dZ[:, vocab_rows]^T H is one product over all rows t.
+
+    ``w_vocab`` may be a float64 array already (it is then used without a
+    copy). Returns float64 ``grad_hidden`` [N, d] and ``grad_w`` [len(vocab_rows), d].
+    """
+    h = as_f64(hidden)
+    w = as_f64(w_vocab)
+    y = as_i64(targets)
+    g = as_f64(grad_logp)
+    gh = np.zeros_like(g) if grad_entropy is None else as_f64(grad_entropy)
+    n, V = h.shape[0], w.shape[0]
+    cols = np.arange(V) if vocab_rows is None else as_i64(vocab_rows)
+    if n and (y.min() < 0 or y.max() >= V):
+        raise ValueError("target out of range [0, V)")
+    grad_hidden = np.empty_like(h)
+    dz_cols = np.empty((n, cols.shape[0]))
+    for r0 in range(0, n, rows_per_block):
+        r1 = min(n, r0 + rows_per_block)
+        z = (h[r0:r1] @ w.T) * float(inv_temperature)
+        dz = _dz_rows(z, y[r0:r1], g[r0:r1], gh[r0:r1], inv_temperature)
+        grad_hidden[r0:r1] = dz @ w
+        dz_cols[r0:r1] = dz[:, cols]
+    return {"grad_hidden": grad_hidden, "grad_w": dz_cols.T @ h}

@@ -13,7 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle.logprobs import token_logprobs, token_logprobs_bwd
+from oracle.logprobs import token_logprobs, token_logprobs_bwd, token_logprobs_bwd_rows
 
 scipy_special = pytest.importorskip("scipy.special")
 
@@ -242,6 +242,33 @@ def test_backward_invariants():
     np.testing.assert_allclose(out["dz"].sum(axis=1), 0.0, atol=1e-13)
     z0 = token_logprobs_bwd(h, w, y, np.zeros(N), None)
     assert not np.any(z0["grad_hidden"]) and not np.any(z0["grad_w"])
+
+
+def test_backward_rows_matches_torch_autograd_fp64():
+    """The row-blocked variant used at full problem sizes (ragged last block,
+    an unsorted subset of vocabulary rows with repeats) against torch fp64
+    autograd of the log-softmax and entropy."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(9)
+    N, d, V = 11, 16, 45
+    h, w = _rand(rng, N, d), _rand(rng, V, d, scale=0.6)
+    y = rng.integers(0, V, N)
+    g, gh = _rand(rng, N), _rand(rng, N)
+    inv_temp = 1.0 / 0.9
+    th = torch.tensor(h, requires_grad=True)
+    tw = torch.tensor(w, requires_grad=True)
+    ls = torch.log_softmax((th @ tw.T) * inv_temp, dim=1)
+    logp = ls[torch.arange(N), torch.tensor(y)]
+    ent = -(ls.exp() * ls).sum(dim=1)
+    ((torch.tensor(g) * logp).sum() + (torch.tensor(gh) * ent).sum()).backward()
+    cols = np.array([44, 0, int(y[3]), 17, 17, 30])
+    out = token_logprobs_bwd_rows(h, w, y, g, gh, inv_temp, vocab_rows=cols, rows_per_block=4)
+    np.testing.assert_allclose(out["grad_hidden"], th.grad.numpy(), atol=1e-12)
+    np.testing.assert_allclose(out["grad_w"], tw.grad.numpy()[cols], atol=1e-12)
+    # All vocabulary rows: each dZ row sums to zero, so grad_w sums to zero over v.
+    full = token_logprobs_bwd_rows(h, w, y, g, None, inv_temp, rows_per_block=3)
+    assert full["grad_w"].shape == (V, d)
+    np.testing.assert_allclose(full["grad_w"].sum(axis=0), 0.0, atol=1e-12)
 
 
 def test_oracle_package_exports():

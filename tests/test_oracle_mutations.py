@@ -110,20 +110,62 @@ LOGPROB_SLIPS = [
      "lse = np.log(np.exp(z - m[:, None]).sum(axis=1))\n    rows"),                    # dropped max shift
 ]
 BACKWARD_SLIPS = [
-    ("dz = float(inv_temperature) * (g[:, None] * (onehot - p)\n"
-     "                                   - gh[:, None] * p * (logp_all + ent[:, None]))",
-     "dz = float(inv_temperature) * (g[:, None] * (onehot - p))"),                    # dropped entropy term
-    ("dz = float(inv_temperature) * (", "dz = 1.0 * ("),                              # dropped temperature
+    ("(g[:, None] * (onehot - p) - gh[:, None] * p * (logp_all + ent[:, None]))",
+     "(g[:, None] * (onehot - p))"),                                                  # dropped entropy term
+    ("return float(inv_temperature) * (", "return 1.0 * ("),                          # dropped temperature
     ("(g[:, None] * (onehot - p)", "(g[:, None] * (p - onehot)"),                    # sign of the softmax term
     ("(logp_all + ent[:, None])", "(logp_all - ent[:, None])"),                      # sign inside the entropy term
     ('"grad_w": dz.T @ h', '"grad_w": dz.T @ (h * 0.5)'),                            # a stray factor on one GEMM
 ]
+# Slips in the row-blocked variant used at full problem sizes.
+BACKWARD_ROWS_SLIPS = [
+    ("dz_cols[r0:r1] = dz[:, cols]", "dz_cols[r0:r1] = dz[:, cols - 1]"),            # wrong vocabulary column
+    ("r1 = min(n, r0 + rows_per_block)\n        z = (h[r0:r1] @ w.T)",
+     "r1 = min(n, r0 + rows_per_block)\n        z = (h[r0:r1] @ w.T) * 0 + (h[r0:r1] @ w.T)[:, ::-1]"),
+                                                                                      # reversed vocabulary order
+    ('"grad_w": dz_cols.T @ h}', '"grad_w": dz_cols.T @ h[::-1]}'),                 # rows of H misaligned with dZ
+    ("grad_hidden[r0:r1] = dz @ w\n", "grad_hidden[r0:r1] = dz @ w * float(inv_temperature)\n"),
+                                                                                      # temperature applied twice
+    ("for r0 in range(0, n, rows_per_block):\n        r1 = min(n, r0 + rows_per_block)\n        z = (h",
+     "for r0 in range(0, n - 1, rows_per_block):\n        r1 = min(n, r0 + rows_per_block)\n        z = (h"),
+                                                                                      # last block dropped
+]
+
+
+def check_backward_rows(mod):
+    """Row-blocked gradients (ragged last block, unsorted vocabulary rows)
+    against central differences of the brute-force loss."""
+    rng = np.random.default_rng(2)
+    N, d, V, inv_temp = 5, 4, 6, 1.0 / 0.9
+    h, w = rng.standard_normal((N, d)), rng.standard_normal((V, d))
+    y, g, gh = rng.integers(0, V, N), rng.standard_normal(N), rng.standard_normal(N)
+    cols = np.array([5, 0, 3])
+    np.seterr(all="raise")
+    try:
+        got = mod.token_logprobs_bwd_rows(h, w, y, g, gh, inv_temp, vocab_rows=cols, rows_per_block=2)
+    finally:
+        np.seterr(all="warn")
+    eps = 1e-6
+
+    def fd(which, idx):
+        xp, xm = (h.copy(), w.copy()), (h.copy(), w.copy())
+        xp[which][idx] += eps
+        xm[which][idx] -= eps
+        lp = _brute_loss(xp[0].tolist(), xp[1].tolist(), y.tolist(), g, gh, inv_temp)
+        lm = _brute_loss(xm[0].tolist(), xm[1].tolist(), y.tolist(), g, gh, inv_temp)
+        return (lp - lm) / (2 * eps)
+
+    want_h = np.array([[fd(0, (t, k)) for k in range(d)] for t in range(N)])
+    want_w = np.array([[fd(1, (v, k)) for k in range(d)] for v in cols])
+    assert np.allclose(got["grad_hidden"], want_h, rtol=1e-6, atol=1e-8), "grad_hidden"
+    assert np.allclose(got["grad_w"], want_w, rtol=1e-6, atol=1e-8), "grad_w rows"
 
 
 def test_unpatched_log_prob_oracle_passes():
     mod = load("logprobs")
     check_forward(mod)
     check_backward(mod)
+    check_backward_rows(mod)
 
 
 @pytest.mark.parametrize("patch", LOGPROB_SLIPS, ids=lambda p: p[1][:40])
@@ -134,6 +176,11 @@ def test_forward_slip_is_caught(patch):
 @pytest.mark.parametrize("patch", BACKWARD_SLIPS, ids=lambda p: p[1][:40])
 def test_backward_slip_is_caught(patch):
     assert fails(check_backward, load("logprobs", patch))
+
+
+@pytest.mark.parametrize("patch", BACKWARD_ROWS_SLIPS, ids=lambda p: p[1][:40])
+def test_backward_rows_slip_is_caught(patch):
+    assert fails(check_backward_rows, load("logprobs", patch))
 
 
 # ------------------------------------------------------------------ filter
