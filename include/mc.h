@@ -152,7 +152,10 @@ mc_status mc_merge_logprob_states(const float* states, int32_t P, int64_t N,
  *   work is queued (about 171,000 rows for V >= 4096; more for smaller V).
  *   Set-up: the first call on each device looks up the array's device address
  *   with that device current and caches it; make that first call before any
- *   stream capture begins.
+ *   stream capture begins. The cached address belongs to the device's context
+ *   as it was at that first call: cudaDeviceReset() on the device invalidates
+ *   it, and this entry point must not be called again on that device in the
+ *   same process afterwards.
  *   Sharing: all calls on a device use the same array and it keeps the last
  *   call's contents (the call clears, on its stream, what must start at zero).
  *   Calls whose work overlaps on the GPU (different streams without ordering

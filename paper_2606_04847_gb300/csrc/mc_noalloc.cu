@@ -30,7 +30,8 @@ std::mutex g_mu;
 void* g_scratch_dev_ptr[kMaxDevices] = {};
 
 // Device address of the scratch on the current device, looked up once per
-// device (with that device current) and cached.
+// device (with that device current) and cached for the life of the process:
+// a cudaDeviceReset() unloads the module and leaves the cached address stale.
 mc_status scratch_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MC_ERR_CUDA;
