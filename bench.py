@@ -14,13 +14,16 @@ formed once before timing (the rollout engine's job, not part of the step).
 
 Rank 0 prints one JSON line. ``value`` = tokens/s over all ranks with inputs
 resident in HBM; ``e2e`` = the same through the C ABI with the step's inputs
-copied from pinned host memory and its per-token / per-sequence results read
-back inside the timed region. Inputs (hidden 1.1 GB, W 2.0 GB) exceed the
-129 MB L2, so no flush is needed between steps. ``--impl reference`` times the
-CPU fp64 oracle instead, on a bounded sample of the same workload.
+copied from pinned host memory and its per-token / per-sequence results and
+grad_hidden read back inside the timed region (grad_w stays on the device for
+the optimizer). Inputs (hidden 1.1 GB, W 2.0 GB) exceed the 129 MB L2, so no
+flush is needed between steps. ``--impl reference`` times the CPU fp64 oracle
+instead, on a bounded sample of the same workload.
 
-Multi-GPU (torchrun): one independent replica per GPU (each rank its own
-batch, weak scaling); the path shards with no data-path collective.
+Multi-GPU (torchrun): one rank per GPU, each on its own batch (weak scaling).
+Forward, filter and grad_hidden need no exchange; for the forward + backward
+step, grad_w (each rank's gradient over its own batch) is all-reduced over
+the ranks with NCCL inside the timed step, as data parallelism requires.
 """
 
 from __future__ import annotations
