@@ -48,6 +48,7 @@ METRIC = "rollout tokens/sec for fused logprob fwd+bwd at 1 GB300; % of bf16 ten
 METRIC_FWD = "rollout tokens/sec for fused logprob fwd + MirrorPop filter at 1 GB300; % of bf16 tensor peak"
 CONFIG_ID = 5  # the fused forward+backward workload the metric names (the default of --config)
 FWD_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fwd_kernel_traffic.json")
+BWD_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "bwd_kernels_traffic.json")
 
 
 def _peaks():
@@ -59,13 +60,17 @@ def _peaks():
     return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
 
 
-def _kernel_source_hash():
-    """Hash of the forward kernel's and its schedule's code, comments and
-    whitespace removed (so that edits to comments keep a capture valid)."""
+FWD_SOURCES = ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu", "mc_schedule.h")  # the forward kernel and its schedule
+BWD_SOURCES = ("mc_gemm.cuh", "mc_ptx.cuh", "mc_bwd.cu", "mc_schedule.h")  # the backward's kernels and schedule
+
+
+def _kernel_source_hash(files=FWD_SOURCES):
+    """Hash of a kernel's and its schedule's code, comments and whitespace
+    removed (so that edits to comments keep a capture valid)."""
     import re
 
     h = hashlib.sha256()
-    for f in ("mc_gemm.cuh", "mc_ptx.cuh", "mc_fwd.cu", "mc_schedule.h"):  # the forward kernel and its schedule
+    for f in files:
         src = open(os.path.join(ROOT, "paper_2606_04847_gb300", "csrc", f)).read()
         src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
         src = re.sub(r"//[^\n]*", " ", src)
@@ -408,6 +413,11 @@ def run_ours(args):
         tj = json.load(open(FWD_TRAFFIC_FILE))
         if tj.get("kernel_source_hash") == _kernel_source_hash() and tj.get("config", 5) == args.config:
             traffic = tj["bytes_per_full_launch"] * (N / tj["full_launch_rows"])
+    traffic_bwd = None
+    if has_bwd and os.path.exists(BWD_TRAFFIC_FILE):
+        tj = json.load(open(BWD_TRAFFIC_FILE))
+        if tj.get("kernel_source_hash") == _kernel_source_hash(BWD_SOURCES) and tj.get("config", 5) == args.config:
+            traffic_bwd = tj["bytes_per_call"] * (kept_rows / tj["rows"])
     step_tflops = (flop_fwd + flop_bwd) * args.steps / (ms / 1e3) / 1e12
 
     # ---------------------------------------------------------------- e2e through the C ABI, host buffers
@@ -575,7 +585,10 @@ def run_ours(args):
                 "note": "achieved = algorithmic 4*N_g*d*V; executed adds the 2*N_g*d*V logit recompute the "
                         "configuration requires",
                 "executed": 1.5 * flop_bwd / (t_bwd / 1e3) / 1e12,
-                "executed_frac": 1.5 * flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf},
+                "executed_frac": 1.5 * flop_bwd / (t_bwd / 1e3) / 1e12 / peak_tf,
+                "traffic": traffic_bwd,
+                "traffic_source": "ncu single-pass capture of the three backward GEMMs of one call, scaled by kept "
+                                  "rows (profiles/bwd_kernels_traffic.json)" if traffic_bwd is not None else None},
             "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)
