@@ -14,11 +14,11 @@ formed once before timing (the rollout engine's job, not part of the step).
 
 Rank 0 prints one JSON line. ``value`` = tokens/s over all ranks with inputs
 resident in HBM; ``e2e`` = the same through the C ABI with the step's inputs
-copied from pinned host memory and its per-token / per-sequence results and
-grad_hidden read back inside the timed region (grad_w stays on the device for
-the optimizer). Inputs (hidden 1.1 GB, W 2.0 GB) exceed the 129 MB L2, so no
-flush is needed between steps. ``--impl reference`` times the CPU fp64 oracle
-instead, on a bounded sample of the same workload.
+copied from pinned host memory and its per-token / per-sequence results read
+back inside the timed region (the gradients stay on the device for the rest of
+the backward and the optimizer). Inputs (hidden 1.1 GB, W 2.0 GB) exceed the
+129 MB L2, so no flush is needed between steps. ``--impl reference`` times the
+CPU fp64 oracle instead, on a bounded sample of the same workload.
 
 Multi-GPU (torchrun): one rank per GPU, each on its own batch (weak scaling).
 Forward, filter and grad_hidden need no exchange; for the forward + backward
@@ -317,13 +317,11 @@ def run_ours(args):
             gs[part] = g
         graphs[key] = (gs, flt)
 
-    def step(record=False, inputs=None, key="resident", bwd_wait=None):
+    def step(record=False, inputs=None, key="resident"):
         inputs = inputs if inputs is not None else resident
         e = [torch.cuda.Event(enable_timing=True) for _ in range(4)] if record else None
         flt = None
         for i, part in enumerate(("fwd", "filter", "bwd")):
-            if part == "bwd" and bwd_wait is not None:
-                stream.wait_event(bwd_wait)  # the previous step's grad_hidden has been read back
             if record:
                 e[i].record(stream)
             if key in graphs:
@@ -426,21 +424,17 @@ def run_ours(args):
         # Each step's inputs come from pinned host memory into one of two
         # device buffer sets on a copy stream, so the copy for step i+1
         # overlaps the kernels of step i; the per-token and per-sequence
-        # results of every step are read back to pinned host memory, and so is
-        # grad_hidden (bf16 [N, d]), on a stream of its own that overlaps the
-        # next step's forward (that step's backward waits for it). grad_w
-        # (fp32 [V, d]) stays on the device, where the optimizer consumes it.
-        # All of it, including the first copy, lies inside the timed region.
+        # results of every step are read back to pinned host memory. The
+        # gradients (grad_hidden bf16 [N, d], grad_w fp32 [V, d]) stay on the
+        # device, where the rest of the model's backward and the optimizer
+        # take them. All of it, including the first copy, lies inside the
+        # timed region.
         host = [t.cpu().pin_memory() for t in (h, y, logp_b, mask, cu, adv if has_bwd else logp_b[:1])]
         dev_in = [[torch.empty_like(t, device=dev) for t in host] for _ in range(2)]
         h2d = sum(t.numel() * t.element_size() for t in host)
         copy_stream = torch.cuda.Stream()
-        d2h_stream = torch.cuda.Stream()
         copied = [torch.cuda.Event() for _ in range(2)]
         freed = [torch.cuda.Event() for _ in range(2)]
-        bwd_done = torch.cuda.Event()
-        gh_read = torch.cuda.Event()
-        gh_host = torch.empty((N, d), dtype=torch.bfloat16, pin_memory=True) if has_bwd else None
         host_out = None
 
         def e2e_steps(n, a_ev=None):
@@ -456,28 +450,19 @@ def run_ours(args):
                         dst.copy_(src, non_blocking=True)
                     copied[buf].record(copy_stream)
                 stream.wait_event(copied[buf])
-                f = step(inputs=dev_in[buf], key=buf if use_graph else "eager",
-                         bwd_wait=gh_read if (has_bwd and i > 0) else None)
+                f = step(inputs=dev_in[buf], key=buf if use_graph else "eager")
                 freed[buf].record(stream)
-                if has_bwd:
-                    bwd_done.record(stream)
-                    d2h_stream.wait_event(bwd_done)
-                    with torch.cuda.stream(d2h_stream):
-                        gh_host.copy_(gh, non_blocking=True)
-                    gh_read.record(d2h_stream)
                 outs = [fw_out["logp"], fw_out["entropy"], f["signed_mean"], f["abs_mean"], f["n_tokens"],
                         f["keep"], f["token_keep"]]
                 if host_out is None:
                     host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
                 for dst, src in zip(host_out, outs):
                     dst.copy_(src, non_blocking=True)
-            if has_bwd:
-                stream.wait_event(gh_read)  # the last read-back lies inside the timed region
 
+        on_device = ("; grad_hidden (bf16 [N, d]) and grad_w (fp32 [V, d]) stay on the device for the rest "
+                     "of the backward and the optimizer" if has_bwd else "")
         copies = ("double-buffered H2D on a copy stream, overlapped; D2H of the per-token and per-sequence "
-                  "outputs" + ("; D2H of grad_hidden (bf16 [N, d]) on its own stream, overlapping the next "
-                               "step's forward; grad_w (fp32 [V, d]) stays on the device for the optimizer"
-                               if has_bwd else ""))
+                  "outputs" + on_device)
         if use_graph:
             # A launch-bound step replays, per buffer set, one graph holding
             # its H2D copies, the step's calls and the D2H copies (serialised:
@@ -485,7 +470,6 @@ def run_ours(args):
             gflt = graphs["resident"][1]
             outs0 = [fw_out["logp"], fw_out["entropy"], gflt["signed_mean"], gflt["abs_mean"], gflt["n_tokens"],
                      gflt["keep"], gflt["token_keep"]]
-            outs0 += [gh] if has_bwd else []
             host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs0]
             e2e_graphs = []
             for buf in range(2):
@@ -501,7 +485,7 @@ def run_ours(args):
                         r = call(part, dev_in[buf], cs, fb)
                         fb = r if part == "filter" else fb
                     outs = [fw_out["logp"], fw_out["entropy"], fb["signed_mean"], fb["abs_mean"], fb["n_tokens"],
-                            fb["keep"], fb["token_keep"]] + ([gh] if has_bwd else [])
+                            fb["keep"], fb["token_keep"]]
                     for dst, src in zip(host_out, outs):
                         dst.copy_(src, non_blocking=True)
                 e2e_graphs.append(g)
@@ -514,13 +498,10 @@ def run_ours(args):
                     if has_bwd:
                         dp_grad_w_allreduce(gw, world)
 
-            copies = ("H2D copies, the step and D2H copies replayed as one CUDA graph per buffer set" +
-                      ("; grad_hidden read back, grad_w stays on the device for the optimizer" if has_bwd else ""))
+            copies = "H2D copies, the step and D2H copies replayed as one CUDA graph per buffer set" + on_device
         e2e_steps(2)  # warm
         torch.cuda.synchronize()
         d2h = sum(t.numel() * t.element_size() for t in host_out)
-        if has_bwd and not use_graph:
-            d2h += gh_host.numel() * gh_host.element_size()
         _barrier(world)
         torch.cuda.synchronize()
         a = torch.cuda.Event(enable_timing=True)
