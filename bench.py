@@ -862,7 +862,7 @@ def main():
     ap.add_argument("--graph", choices=["auto", "on", "off"], default="auto",
                     help="replay each call of the step as a CUDA graph (auto: when a step is launch-bound)")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--cpu-rows", type=int, default=384)
+    ap.add_argument("--cpu-rows", type=int, default=512)
     ap.add_argument("--ref-rows", type=int, default=64)
     ap.add_argument("--case", choices=["step", "fwd", "bwd", "filter", "loss", "stream", "next", "advantage"],
                     default="step",
