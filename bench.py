@@ -770,7 +770,8 @@ def run_advantage(args):
 def run_case(args):
     """One call of the path, `--launches` times, for ncu captures (no timing printed
     beyond a one-line summary): --case fwd|bwd|filter|loss on the first `--rows`
-    tokens of the workload (0 = all)."""
+    tokens of the `--config` workload (0 = all; bwd needs config 5, the one with
+    advantage weights)."""
     from paper_2606_04847_gb300 import build as mcbuild
     from paper_2606_04847_gb300 import mc, workloads
 
@@ -783,15 +784,19 @@ def run_case(args):
     torch.cuda.set_device(0)
     if not os.path.exists(mc.lib_path()):
         mcbuild.build()
-    spec = workloads.spec_for(CONFIG_ID)
-    wl = workloads.build(spec, "cuda")
+    spec = workloads.spec_for(args.config)
+    if args.case in ("bwd", "loss") and not spec.advantages:
+        raise SystemExit(f"--case {args.case} needs a workload with advantage weights (--config 5)")
+    # A --rows case draws only those rows (one sequence of the configuration's
+    # shapes and distributions), so that a small capture holds little memory.
+    wl = workloads.build(spec, "cuda", lengths=[args.rows] if args.rows > 0 else None)
     R = wl.N if args.rows <= 0 else min(args.rows, wl.N)
     h, w, y = wl.hidden[:R].contiguous(), wl.w_vocab, wl.targets[:R].contiguous()
     fw = mc.token_logprobs(h, w, y)
     cu = torch.tensor([0, R], dtype=torch.int64, device="cuda")
     lb = (fw["logp"] + wl.gap[:R]).contiguous()
     flt = mc.seq_ratio_filter(fw["logp"], lb, None, cu, spec.delta, spec.delta)
-    adv = wl.advantages[:R].contiguous()
+    adv = wl.advantages[:R].contiguous() if spec.advantages else None
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(args.launches):
@@ -805,7 +810,7 @@ def run_case(args):
         else:  # every row live, so the capture does not depend on whether the filter keeps this slice
             mc.token_logprobs_bwd(h, w, y, fw["lse"], fw["entropy"], adv, None)
     torch.cuda.synchronize()
-    print(json.dumps({"case": args.case, "rows": R, "launches": args.launches,
+    print(json.dumps({"case": args.case, "config": args.config, "rows": R, "launches": args.launches,
                       "wall_ms_per_launch": (time.perf_counter() - t0) * 1e3 / args.launches}))
 
 
