@@ -231,6 +231,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.part = reinterpret_cast<float*>(ws + L.part_off);
   a.zy = reinterpret_cast<float*>(ws + L.zy_off);
   a.ws_status = reinterpret_cast<int32_t*>(ws + L.status_off);
+  a.wave_ctr = reinterpret_cast<unsigned int*>(ws + L.status_off + 64);
   a.logp = logp;
   a.entropy = entropy;
   a.lse = lse;
@@ -243,7 +244,7 @@ mc_status queue_forward(const void* hidden, const void* w_vocab, const int32_t* 
   a.halves = (a.wide && 2 * a.splits <= max_splits(V)) ? 2 : 1;
   a.v_offset = v_offset;
   a.state = state;
-  cudaError_t e = cudaMemsetAsync(a.ws_status, 0, sizeof(int32_t), s);
+  cudaError_t e = cudaMemsetAsync(ws + L.status_off, 0, 128, s);  // status word and wave gate counter
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   e = mc::launch_forward(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "forward launch");

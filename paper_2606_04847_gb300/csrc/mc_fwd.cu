@@ -253,7 +253,21 @@ cudaError_t run_forward_gemm(const FwdArgs& a, const Schedule& sch, const FwdPar
   if (e != cudaSuccess) return e;
   const int units = sch.m_blocks * sch.splits;
   const int grid = units < a.grid ? units : a.grid;
-  kern<<<grid, TileFor<Epi, MS>::THREADS, smem, stream>>>(a.tm_hidden, a.tm_w, sch, ep, a.timeout_ns, a.ws_status);
+  // Cooperative launch: the wave gate needs every CTA resident (one per SM).
+  Schedule gated = sch;
+  gated.wave_ctr = a.wave_ctr;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(TileFor<Epi, MS>::THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, a.tm_hidden, a.tm_w, gated, ep, a.timeout_ns, a.ws_status);
+  if (e != cudaSuccess) return e;
   return launched();
 }
 

@@ -122,6 +122,15 @@ struct Schedule {
   // n_group tiles instead of ~grid/n_tiles x all tiles. A long-K GEMM re-reads
   // both operands once per wave; this shape reads fewer bytes per wave.
   int n_group = 0;
+  // Optional wave gate (a counter that is zero at launch; the launch must be
+  // cooperative, so that every CTA is resident). Each CTA's producer raises
+  // it after issuing a unit's loads and, before its k-th unit (k >= 1), waits
+  // until min(k * gridDim.x, units) units have been issued: no CTA starts a
+  // wave before every CTA has finished the one before. The CTAs that share a
+  // unit's B tiles then read each tile within a few tiles of one another, and
+  // the tile is still in L2 for all of them; without the gate they drift
+  // apart over many waves and re-read B from HBM.
+  unsigned int* wave_ctr = nullptr;
 
   __device__ __forceinline__ int units() const { return m_blocks * splits; }
   __device__ __forceinline__ void unit(int u, int& mb, int& split, int& t0, int& t1) const {
@@ -254,7 +263,14 @@ __global__ void __launch_bounds__(TileFor<Epi, MS>::THREADS, 1)
       tma_prefetch_desc(&tmB);
       uint32_t it = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      for (int u = blockIdx.x, wave = 0; u < n_units && ok; u += gridDim.x, ++wave) {
+        if (sch.wave_ctr != nullptr && wave > 0) {
+          const unsigned need = min(static_cast<unsigned>(wave) * gridDim.x, static_cast<unsigned>(n_units));
+          if (!counter_wait_geq(sch.wave_ctr, need, abort, timeout_ns, dev_status)) {
+            ok = false;
+            break;
+          }
+        }
         int mb, split, t0, t1;
         sch.unit(u, mb, split, t0, t1);
         const int row0 = mb * C::TBM;
@@ -289,6 +305,7 @@ __global__ void __launch_bounds__(TileFor<Epi, MS>::THREADS, 1)
             ++it;
           }
         }
+        if (sch.wave_ctr != nullptr && ok) atomicAdd(sch.wave_ctr, 1u);
       }
       // Let every load this thread issued land before the CTA can exit.
       const uint32_t last = it < C::STAGES ? it : C::STAGES;

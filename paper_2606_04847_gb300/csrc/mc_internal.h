@@ -33,6 +33,7 @@ struct FwdArgs {
   float* part;            // workspace: [3][splits * halves][n_pad]
   float* zy;              // workspace: [n_pad]
   int32_t* ws_status;     // workspace: internal status word (zeroed by the caller)
+  unsigned int* wave_ctr; // workspace: the projection's wave gate counter (zeroed by the caller)
   float* logp;
   float* entropy;
   float* lse;

@@ -80,6 +80,29 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// Bounded wait until *ctr >= need, a counter that other CTAs of the same
+// (cooperatively launched) grid raise. Same give-up rules as mbar_wait.
+__device__ __forceinline__ bool counter_wait_geq(const unsigned int* ctr, unsigned int need, volatile int* abort,
+                                                 uint64_t timeout_ns, int32_t* dev_status) {
+  auto load = [&] {
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    return v;
+  };
+  if (load() >= need) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(64);
+    if (load() >= need) return true;
+    if (abort != nullptr && *abort) return false;
+    if ((it & 15u) == 0u && (globaltimer_ns() - t0 > timeout_ns || it > (1u << 30))) {
+      if (abort != nullptr) *abort = 1;
+      if (dev_status) atomicOr(dev_status, MC_DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+
 // ---------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
