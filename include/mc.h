@@ -316,11 +316,13 @@ mc_status mc_prime_echo_advantages(const float* scores, const uint8_t* success, 
                                    mc_stream_t stream);
 
 /* ------------------------------------------------------------------------
- * Self-test of the bounded device wait used by every pipelined kernel: one
- * CTA waits on a shared-memory barrier that nothing ever signals, gives up
- * after `timeout_ns` nanoseconds (1e6 <= timeout_ns <= 1e10), sets
- * MC_DEV_TIMEOUT in *dev_status and returns. Exercises the failure path
- * without faulting or hanging the GPU. (No counterpart in the paper.)
+ * Self-test of the bounded device waits used by every pipelined kernel: one
+ * CTA waits on a shared-memory barrier that nothing ever signals and, in a
+ * second warp, on a global counter that nothing ever raises (the wait of the
+ * GEMMs' wave gate); each gives up after `timeout_ns` nanoseconds
+ * (1e6 <= timeout_ns <= 1e10), sets MC_DEV_TIMEOUT in *dev_status and
+ * returns. Exercises the failure path without faulting or hanging the GPU.
+ * (No counterpart in the paper.)
  * ------------------------------------------------------------------------ */
 mc_status mc_selftest_bounded_wait(int32_t* dev_status, int64_t timeout_ns, mc_stream_t stream);
 

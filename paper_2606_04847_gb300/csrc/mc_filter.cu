@@ -158,8 +158,12 @@ __global__ void __launch_bounds__(kFilterThreads) seq_filter_kernel(FilterArgs p
   }
 }
 
-// Waits on a barrier nothing arrives at, through the same bounded wait the
-// pipelined kernels use, and must come back with MC_DEV_TIMEOUT set.
+// A global counter nothing ever raises (zero for the life of the module).
+__device__ unsigned int g_selftest_counter;
+
+// Waits, through the two bounded waits the pipelined kernels use, on a
+// barrier nothing arrives at (warp 0) and on a global counter nothing raises
+// (warp 1, the wave gate's wait); each must give up and set MC_DEV_TIMEOUT.
 __global__ void selftest_wait_kernel(int32_t* dev_status, uint64_t timeout_ns) {
   __shared__ uint64_t bar;
   __shared__ int abort_flag;
@@ -170,6 +174,7 @@ __global__ void selftest_wait_kernel(int32_t* dev_status, uint64_t timeout_ns) {
   }
   __syncthreads();
   if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, timeout_ns, dev_status);
+  if (threadIdx.x == 32) counter_wait_geq(&g_selftest_counter, 1u, nullptr, timeout_ns, dev_status);
 }
 
 }  // namespace
@@ -195,7 +200,7 @@ cudaError_t launch_filter(const FilterArgs& a, cudaStream_t stream) {
 }
 
 cudaError_t launch_selftest_wait(int32_t* dev_status, uint64_t timeout_ns, cudaStream_t stream) {
-  selftest_wait_kernel<<<1, 32, 0, stream>>>(dev_status, timeout_ns);
+  selftest_wait_kernel<<<1, 64, 0, stream>>>(dev_status, timeout_ns);
   return launched();
 }
 

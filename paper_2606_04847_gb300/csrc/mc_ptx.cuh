@@ -95,7 +95,8 @@ __device__ __forceinline__ bool counter_wait_geq(const unsigned int* ctr, unsign
     __nanosleep(64);
     if (load() >= need) return true;
     if (abort != nullptr && *abort) return false;
-    if ((it & 15u) == 0u && (globaltimer_ns() - t0 > timeout_ns || it > (1u << 30))) {
+    // Each poll sleeps ~64 ns, so 2^27 polls back up the clock at ~10 s.
+    if ((it & 15u) == 0u && (globaltimer_ns() - t0 > timeout_ns || it > (1u << 27))) {
       if (abort != nullptr) *abort = 1;
       if (dev_status) atomicOr(dev_status, MC_DEV_TIMEOUT);
       return false;
