@@ -30,6 +30,8 @@
 // round-robin to the persistent CTAs (unit u -> CTA u % gridDim.x), so the
 // CTAs running at the same time share a few row blocks (A stays in L2) and
 // sweep the same B tiles together (B is read from HBM about once per wave).
+// The library launches every GEMM cooperatively with a wave gate
+// (Schedule::wave_ctr) that keeps the waves in step.
 // Within a unit the tiles run in order, so an epilogue can carry per-row
 // state across them (the forward's online softmax).
 //
