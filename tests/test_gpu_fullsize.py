@@ -18,6 +18,8 @@ times (whole batches through the C ABI, default workspaces).
   statistics and keep decisions, and 256 of their grad_hidden rows; grad_w,
   which sums over all ~90k kept rows, is checked through identities that hold
   at any size: <grad_hidden, H> = <grad_w, W> and sum_v grad_w[v, :] = 0.
+* the 27B-class batch end to end through the filter with its per-turn loss
+  mask: the oracle recomputes a kept and a dropped sequence whole.
 """
 
 import numpy as np
@@ -278,6 +280,48 @@ def test_chain_full_size_9b():
     col = gw.double().sum(dim=0)
     scale = gw.double().abs().sum(dim=0)
     assert (col.abs() <= 1e-3 * scale + 1e-6).all()
+
+
+def test_chain_27b_whole_sequences():
+    """27B-class batch (d = 5120, multi-turn sequences, the prompt tokens of
+    every turn masked out of the loss): forward over all 595k tokens, then the
+    MirrorPop filter with the per-turn loss mask. The oracle recomputes the
+    shortest kept and the shortest dropped sequence whole from their hidden
+    states: every log-prob, the masked token count L_i, the Eq. 20 statistic
+    and the Eq. 21 decision."""
+    spec = workloads.spec_for(4)
+    wl = workloads.build(spec, "cuda")
+    fw = mc.token_logprobs(wl.hidden, wl.w_vocab, wl.targets)
+    lb = fw["logp"] + wl.gap
+    flt = mc.seq_ratio_filter(fw["logp"], lb, wl.loss_mask, wl.cu_seqlens, spec.delta, spec.delta)
+    torch.cuda.synchronize()
+    cu = np_(wl.cu_seqlens)
+    gap = np_(wl.gap)[cu[:-1]]
+    lens = np.diff(cu)
+    far = np.abs(np.abs(gap) - spec.delta) > 0.02
+    kept_i = min(np.nonzero(far & (np.abs(gap) < spec.delta))[0], key=lambda i: lens[i])
+    drop_i = min(np.nonzero(far & (np.abs(gap) > spec.delta))[0], key=lambda i: lens[i])
+    seqs = [kept_i, drop_i]
+    rows = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in seqs])
+    ridx = torch.from_numpy(rows).cuda()
+    w64 = wl.w_vocab.cpu().double().numpy()
+    ref_f = oracle.token_logprobs(wl.hidden[ridx].cpu(), w64, wl.targets[ridx].cpu(), rows_per_block=TILE_ROWS)
+    del w64
+    assert_close_abs(np_(fw["logp"][ridx]), ref_f["logp"], TOL_LOGP, "27B logp")
+    assert_close_abs(np_(fw["entropy"][ridx]), ref_f["entropy"], TOL_ENT, "27B entropy")
+    sub_cu = np.concatenate([[0], np.cumsum(lens[seqs])])
+    mask_rows = np_(wl.loss_mask[ridx])
+    ref_flt = oracle.seq_ratio_filter(ref_f["logp"], ref_f["logp"] + np_(wl.gap[ridx]).astype(np.float64),
+                                      mask_rows, sub_cu, float(np.float32(spec.delta)))
+    assert list(ref_flt["keep"]) == [1, 0]
+    assert 0 < ref_flt["n_tokens"][0] < lens[kept_i]  # the prompt tokens of every turn are masked out
+    np.testing.assert_array_equal(np_(flt["n_tokens"])[seqs], ref_flt["n_tokens"])
+    dlogp = np.abs(np_(fw["logp"][ridx]) - ref_f["logp"])
+    band = MASK_BAND + np.array([dlogp[sub_cu[k]:sub_cu[k + 1]].mean() for k in range(2)])
+    assert_masks_match(np_(flt["keep"])[seqs], ref_flt["keep"], ref_flt["abs_mean"], spec.delta, band, "27B keep")
+    assert_close_rel(np.exp(np_(flt["abs_mean"])[seqs]), np.exp(ref_flt["abs_mean"]), TOL_RATIO, "27B e^A")
+    tk = np_(flt["token_keep"][ridx]).astype(bool)
+    np.testing.assert_array_equal(tk, ref_flt["token_keep"].astype(bool))
 
 
 def test_full_size_step_is_bitwise_reproducible():
