@@ -19,7 +19,8 @@ times (whole batches through the C ABI, default workspaces).
   which sums over all ~90k kept rows, is checked through identities that hold
   at any size: <grad_hidden, H> = <grad_w, W> and sum_v grad_w[v, :] = 0.
 * the 27B-class batch end to end through the filter with its per-turn loss
-  mask: the oracle recomputes a kept and a dropped sequence whole.
+  mask, and the mid and 9B-class forward workloads end to end through the
+  filter: the oracle recomputes a kept and a dropped sequence whole.
 """
 
 import numpy as np
@@ -322,6 +323,49 @@ def test_chain_27b_whole_sequences():
     assert_close_rel(np.exp(np_(flt["abs_mean"])[seqs]), np.exp(ref_flt["abs_mean"]), TOL_RATIO, "27B e^A")
     tk = np_(flt["token_keep"][ridx]).astype(bool)
     np.testing.assert_array_equal(tk, ref_flt["token_keep"].astype(bool))
+
+
+@pytest.mark.parametrize("config", [2, 3])
+def test_chain_forward_workloads_whole_sequences(config):
+    """The mid (per-token behaviour gap on 10 % of sequences) and 9B-class
+    forward workloads end to end: forward over the whole batch, then the
+    filter; the oracle recomputes one kept and one dropped sequence whole
+    (chosen from the synthetic gap: with logp_behaviour = logp_policy + gap,
+    A_i is the mean |gap| over the sequence's loss-masked tokens)."""
+    spec = workloads.spec_for(config)
+    wl = workloads.build(spec, "cuda")
+    fw = mc.token_logprobs(wl.hidden, wl.w_vocab, wl.targets)
+    lb = fw["logp"] + wl.gap
+    flt = mc.seq_ratio_filter(fw["logp"], lb, wl.loss_mask, wl.cu_seqlens, spec.delta, spec.delta)
+    torch.cuda.synchronize()
+    cu = np_(wl.cu_seqlens)
+    lens = np.diff(cu)
+    gap, m = np.abs(np_(wl.gap).astype(np.float64)), np_(wl.loss_mask).astype(bool)
+    a_gap = np.array([gap[cu[i]:cu[i + 1]][m[cu[i]:cu[i + 1]]].mean() for i in range(wl.B)])
+    far = np.abs(a_gap - spec.delta) > 0.01
+    kept_i = min(np.nonzero(far & (a_gap < spec.delta))[0], key=lambda i: lens[i])
+    drop_i = min(np.nonzero(far & (a_gap > spec.delta))[0], key=lambda i: lens[i])
+    seqs = [kept_i, drop_i]
+    rows = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in seqs])
+    ridx = torch.from_numpy(rows).cuda()
+    w64 = wl.w_vocab.cpu().double().numpy()
+    ref_f = oracle.token_logprobs(wl.hidden[ridx].cpu(), w64, wl.targets[ridx].cpu(), rows_per_block=TILE_ROWS)
+    del w64
+    assert_close_abs(np_(fw["logp"][ridx]), ref_f["logp"], TOL_LOGP, f"config {config} logp")
+    assert_close_abs(np_(fw["entropy"][ridx]), ref_f["entropy"], TOL_ENT, f"config {config} entropy")
+    sub_cu = np.concatenate([[0], np.cumsum(lens[seqs])])
+    ref_flt = oracle.seq_ratio_filter(ref_f["logp"], ref_f["logp"] + np_(wl.gap[ridx]).astype(np.float64),
+                                      np_(wl.loss_mask[ridx]), sub_cu, float(np.float32(spec.delta)),
+                                      float(np.float32(spec.delta)))
+    assert list(ref_flt["keep"]) == [1, 0]
+    np.testing.assert_array_equal(np_(flt["n_tokens"])[seqs], ref_flt["n_tokens"])
+    dlogp = np.abs(np_(fw["logp"][ridx]) - ref_f["logp"])
+    band = MASK_BAND + np.array([dlogp[sub_cu[k]:sub_cu[k + 1]].mean() for k in range(2)])
+    assert_masks_match(np_(flt["keep"])[seqs], ref_flt["keep"], ref_flt["abs_mean"], spec.delta, band, "keep")
+    assert_masks_match(np_(flt["keep_vanilla"])[seqs], ref_flt["keep_vanilla"], np.abs(ref_flt["signed_mean"]),
+                       spec.delta, band, "keep_vanilla")
+    assert_close_rel(np.exp(np_(flt["abs_mean"])[seqs]), np.exp(ref_flt["abs_mean"]), TOL_RATIO, "e^A")
+    assert_close_rel(np.exp(np_(flt["signed_mean"])[seqs]), np.exp(ref_flt["signed_mean"]), TOL_RATIO, "e^S")
 
 
 def test_full_size_step_is_bitwise_reproducible():
