@@ -358,6 +358,10 @@ def test_chain_forward_workloads_whole_sequences(config):
                                       np_(wl.loss_mask[ridx]), sub_cu, float(np.float32(spec.delta)),
                                       float(np.float32(spec.delta)))
     assert list(ref_flt["keep"]) == [1, 0]
+    if config == 2:
+        # A per-token gap of mean ~0: the signed statistic cancels (Vanilla
+        # keeps the sequence) while the absolute one does not (MirrorPop drops it).
+        assert ref_flt["keep_vanilla"][1] == 1
     np.testing.assert_array_equal(np_(flt["n_tokens"])[seqs], ref_flt["n_tokens"])
     dlogp = np.abs(np_(fw["logp"][ridx]) - ref_f["logp"])
     band = MASK_BAND + np.array([dlogp[sub_cu[k]:sub_cu[k + 1]].mean() for k in range(2)])
