@@ -37,11 +37,8 @@ inline int concurrent_units(int sms) { return sms; }
 // to the fewest splits. W is read from HBM once per wave, so fewer splits
 // (fewer, larger waves) stream it fewer times: under the GPU's power cap the
 // DRAM energy saved buys more SM clock than a slightly longer tail costs.
-// Past ~100 MB of rows per wave the hidden rows no longer stay in L2, and
-// the W tiles that the splits of a wave stream need the rest of it: at
-// d = 5120 a budget of 56 MB (7 splits) halved the forward's DRAM reads
-// against 80 MB (5 splits) at the same speed.
-constexpr double kWaveRowBytes = 56.0 * (1 << 20);
+// Past ~100 MB of rows per wave the hidden rows no longer stay in L2.
+constexpr double kWaveRowBytes = 80.0 * (1 << 20);
 constexpr double kPathSlack = 1.015;
 
 inline int choose_splits(long long m_blocks, int n_tiles, int conc, int rb, int d) {

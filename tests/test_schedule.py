@@ -81,7 +81,7 @@ def test_splits_of_the_configured_workloads(splits):
         "9B fwd+bwd forward (128,236 tokens)": ((501, 970, 152, 256, 4096), 6),
         "9B fwd+bwd dZ (83,586 kept tokens)": ((327, 970, 152, 256, 4096), 6),
         "9B forward (143,463 tokens)": ((561, 970, 152, 256, 4096), 7),
-        "27B forward (595,356 tokens)": ((2326, 970, 152, 256, 5120), 7),
+        "27B forward (595,356 tokens)": ((2326, 970, 152, 256, 5120), 5),
         "mid forward (32,768 tokens, V = 151,936)": ((128, 594, 152, 256, 4096), 7),
         "one of 4 vocabulary slices (62,080 rows)": ((501, 243, 152, 256, 4096), 6),
     }
