@@ -9,7 +9,12 @@
  * finished. The library allocates no device memory: scratch comes in through
  * `workspace` arguments sized by the matching *_workspace_size() query.
  *
- * Calls are stream-ordered and asynchronous. Errors that can be found on the
+ * Calls are stream-ordered and asynchronous. The tensor-core kernels of the
+ * forward and backward are persistent cooperative launches, one CTA per SM
+ * with every CTA resident (the CTAs keep their waves in step through a
+ * bounded wait on a counter in the caller's workspace): such a kernel starts
+ * once the whole GPU is free and does not share it with concurrent kernels.
+ * Errors that can be found on the
  * host (null or misaligned pointers, bad sizes, a workspace that is too small,
  * no sm_103 device) return a non-zero mc_status synchronously and queue no
  * work. Errors found on the device (a target outside [0, V), a bounded wait
