@@ -13,7 +13,7 @@
  * forward and backward are persistent cooperative launches, one CTA per SM
  * with every CTA resident (the CTAs keep their waves in step through a
  * bounded wait on a counter in the caller's workspace): such a kernel starts
- * once the whole GPU is free and does not share it with concurrent kernels.
+ * only when every SM has room for one of its CTAs at once.
  * Errors that can be found on the
  * host (null or misaligned pointers, bad sizes, a workspace that is too small,
  * no sm_103 device) return a non-zero mc_status synchronously and queue no
