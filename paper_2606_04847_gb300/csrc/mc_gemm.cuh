@@ -94,7 +94,8 @@ constexpr size_t kEpiStageOffset = (size_t(NUM_STAGES) * STAGE_BYTES + sizeof(Ge
 // for two warp groups per 128-row sub-block of a 256-row tile, each draining
 // half of the tile's 256 columns (16 epilogue warps: twice the warps hiding
 // TMEM-load and arithmetic latency while the MMAs wait for the drain). The
-// engine then calls `epi.set_half(h)` once, h = the warp's column half.
+// engine then calls `epi.set_half(h)` once, h = the warp's column half. Their
+// staging buffers (kStageBytes each) must fit beside the operand ring.
 template <class E, class = void>
 struct EpiColumnHalves {
   static constexpr int value = 1;
@@ -211,7 +212,6 @@ __global__ void __launch_bounds__(TileFor<Epi, MS>::THREADS, 1)
                     const uint64_t timeout_ns, int32_t* dev_status) {
   using C = TileFor<Epi, MS>;
   static_assert(C::template smem_bytes<Epi>() <= 227 * 1024, "shared memory of one CTA exceeded");
-  static_assert(C::HALVES == 1 || EpiStage<Epi>::bytes == 0, "column halves are for epilogues without staging");
   Schedule sch = sch_in;
   long long rows_eff = -1;
   bool k_nonempty = true;
